@@ -1,0 +1,296 @@
+"""Benchmark of the action-expert tick (one step = one tick of the whole hot
+path: embed, 32 x [RMSNorm+QKV, Eq. 1 attention, W_o, RMSNorm+SwiGLU, W_d],
+head) on synthetic seeded inputs, printed as one JSON line.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl fsx|reference]
+
+Default workload: bf16_b1_l224 (B=1 vehicle, 224 cached backbone tokens per
+layer = 64 instruction + 40 frames x 4, bf16 weights/cache/frames, 32 layers).
+value = vehicle-ticks/s over all ranks (weak scaling: every rank runs its own
+vehicles; the path has no cross-vehicle exchange). Inputs are resident in HBM
+when the timed region starts; weights (675 MB) plus cache exceed the 129 MB L2,
+so no flush is needed between ticks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "vehicle-ticks/s (1e6 / us-per-tick x B) of the action-expert tick"
+UNIT = "vehicle-ticks/s"
+FALLBACK_HBM_GBS = 6800.0
+KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down"]
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--workload", default="bf16_b1_l224")
+    ap.add_argument("--impl", default="fsx", choices=["fsx", "reference"])
+    ap.add_argument("--kernel-class", default="qkv", choices=KCLASS_NAMES)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            p = json.load(fh)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def workload_info(name):
+    from paper_2607_15621_gb300 import synth
+    spec = synth.WORKLOADS[name]
+    lengths = synth.cache_lengths(name, 0)
+    return spec, lengths
+
+
+def algorithmic_bytes(dims, lengths, cache_dtype, weight_bytes):
+    """Per tick: expert weights once + every vehicle's cache rows once at every layer."""
+    elem = 2 if cache_dtype == "bf16" else 4
+    kv = int(np.sum(lengths)) * dims.n_layers * 2 * dims.hd * elem
+    return weight_bytes + kv, kv
+
+
+def start_clock_sampler(path, index):
+    try:
+        fh = open(path, "w")
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        proc = subprocess.Popen(["nvidia-smi", f"--id={index}", f"--query-gpu={q}", "--format=csv,noheader,nounits",
+                                 "-lms", "200"], stdout=fh, stderr=subprocess.DEVNULL)
+        return proc, fh
+    except Exception:
+        return None, None
+
+
+def stop_clock_sampler(proc, fh, path):
+    if proc is None:
+        return None
+    proc.terminate()
+    try:
+        proc.wait(timeout=5)
+    except Exception:
+        proc.kill()
+    fh.close()
+    sm, smax, reasons = [], [], set()
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    with open(path) as f:
+        for line in f:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+    if not sm:
+        return None
+    return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+            "samples": len(sm)}
+
+
+def cpu_baseline(name, seconds):
+    """The fp64 oracle as it stands, on the host cores, on vehicle 0 of the workload."""
+    from oracle import fsx_oracle
+    from paper_2607_15621_gb300 import synth
+    spec, lengths = workload_info(name)
+    dims = synth.EXPERT
+    w = synth.make_weights(dims, 0, spec["dtype"])
+    k, v, off = synth.make_cache(dims, lengths[:1], 0, spec["dtype"])
+    kn = [t.float().numpy() for t in k]
+    vn = [t.float().numpy() for t in v]
+    fr = synth.make_frames(dims, 1, 0, spec["dtype"]).double().numpy()
+    n, t0 = 0, time.perf_counter()
+    while True:
+        fsx_oracle.expert_tick(w, kn, vn, off, fr, dims.n_heads, dims.head_dim, dims.n_waypoints)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or n >= 1000:
+            break
+    return {"value": n / el, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{n} full 32-layer fp64 ticks of vehicle 0 of {name} (L={int(lengths[0])}) in {el:.1f} s"}
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    spec, lengths = workload_info(args.workload)
+    cb = cpu_baseline(args.workload, max(1.0, min(args.cpu_seconds, 60.0)))
+    line = {"impl": "reference", "metric": METRIC, "value": cb["value"], "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / cb["value"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded)",
+            "config": {"workload": args.workload, "B": 1, "cache_len": int(lengths[0]), "layers": 32},
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    import torch
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from paper_2607_15621_gb300 import fsx, synth
+    spec, lengths = workload_info(args.workload)
+    dims = synth.EXPERT
+    dtype = spec["dtype"]
+    B = len(lengths)
+    w = synth.make_weights(dims, 0, dtype)
+    k, v, off = synth.make_cache(dims, lengths, 0, dtype, device=dev)
+    frames = synth.make_frames(dims, B, 0, dtype, device=dev)
+    offsets = torch.as_tensor(off, device=dev)
+    out = torch.empty(B, dims.n_waypoints, 2, device=dev)
+    ex = fsx.Expert(dims, w, B, int(off[-1]), dtype, dtype, device=local)
+    del w
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(max(args.warmup, 3)):
+        ex.tick(k, v, offsets, frames, out, stream)
+    torch.cuda.synchronize()
+    if ex.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during warm-up")
+
+    clock_path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")
+    os.makedirs(os.path.dirname(clock_path), exist_ok=True)
+    proc, fh = start_clock_sampler(clock_path, local)
+    time.sleep(0.5)
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        ex.tick(k, v, offsets, frames, out, stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    ms = e0.elapsed_time(e1)
+    clocks = stop_clock_sampler(proc, fh, clock_path)
+    if ex.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during the timed region")
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_per_step = ms / args.steps
+    value = world * B * args.steps / (ms / 1e3)
+
+    # ---- end to end through the host-buffer entry point (copies inside the timed region)
+    frames_h = frames.cpu().pin_memory()
+    off_h = torch.as_tensor(off).pin_memory()
+    out_h = torch.empty(B, dims.n_waypoints, 2).pin_memory()
+    for _ in range(3):
+        ex.tick_host(k, v, off_h.numpy(), frames_h, out_h.numpy(), stream)
+    barrier()
+    e2e_steps = max(1, args.steps // 2)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        ex.tick_host(k, v, off_h.numpy(), frames_h, out_h.numpy(), stream)
+    e2e_s = time.perf_counter() - t0
+    barrier()
+    h2d = frames_h.numel() * frames_h.element_size() + off_h.numel() * 8
+    d2h = out_h.numel() * 4
+
+    # ---- dominant kernel: CUDA events around its launches inside the replayed tick graph
+    kclass = args.kernel_class
+    ex.set_kernel_timing(True, kclass)
+    kt_ms, kt_n = [], 0
+    for i in range(max(args.steps // 4, 5) + 2):
+        ex.tick(k, v, offsets, frames, out, stream)
+        t, n = ex.kernel_time()
+        if i >= 2:
+            kt_ms.append(t)
+            kt_n = n
+    ex.set_kernel_timing(False, kclass)
+    per_launch_s = statistics.mean(kt_ms) / kt_n / 1e3
+    d, hd, f = dims.d_model, dims.hd, dims.d_ff
+    M = B * dims.n_tok
+    unit_bytes = {  # algorithmic bytes of one launch (one layer): weights + activations in/out
+        "qkv": 3 * hd * d * 2 + M * d * 4 + M * 3 * hd * 2,
+        "out_proj": d * hd * 2 + M * hd * 2 + 2 * M * d * 4,
+        "gate_up": 2 * f * d * 2 + M * d * 4 + M * f * 2,
+        "down": d * f * 2 + M * f * 2 + 2 * M * d * 4,
+        "attention": int(np.sum(lengths)) * 2 * hd * (2 if dtype == "bf16" else 4) + M * 3 * hd * 2 + M * hd * 2,
+    }[kclass]
+    hbm, peak_kind = peaks()
+    achieved = unit_bytes / per_launch_s / 1e9
+    tick_bytes, kv_bytes = algorithmic_bytes(dims, lengths, dtype, ex.weight_bytes())
+    tick_gbs = tick_bytes / (ms_per_step / 1e3) / 1e9
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": max(args.warmup, 3), "ms_per_step": ms_per_step, "us_per_tick": ms_per_step * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f16 (fp32 accumulate)",
+        "data": "synthetic (seeded N(0,1) cache/frames, N(0,1/fan_in) weights)",
+        "config": {"workload": args.workload, "B": B, "cache_len": [int(x) for x in lengths[:4]],
+                   "layers": dims.n_layers, "d_model": dims.d_model, "tokens_per_vehicle": dims.n_tok,
+                   "l2": "inputs larger than L2 (weights + cache per tick exceed 129 MB)",
+                   "parallelism": f"replicas x{world}"},
+        "gpu_launches": ex.launches(B) * args.steps,
+        "roofline": {"bound": "hbm", "kernel": kclass, "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm, "traffic": None, "peak_source": peak_kind,
+                     "bytes_per_launch": unit_bytes, "launch_us": per_launch_s * 1e6},
+        "tick_roofline": {"bytes_per_tick": tick_bytes, "kv_bytes_per_tick": kv_bytes, "achieved_gbs": tick_gbs,
+                          "frac_of_measured_hbm": tick_gbs / hbm, "frac_of_8tbs": tick_gbs / 8000.0},
+        "e2e": {"value": world * B * e2e_steps / e2e_s, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h)},
+        "clocks": clocks,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.workload, args.cpu_seconds)
+    ex.close()
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,186 @@
+/*
+ * fsx.h -- C ABI of the GB300 action-expert tick.
+ *
+ * The fast system of an asynchronous fast-slow driving agent ("Think at 5 Hz,
+ * Act at 20 Hz", Sec. 3.1 and Sec. 3.3): a 32-layer action expert whose tokens,
+ * at every layer l, attend over the concatenation of the frozen backbone's
+ * layer-l KV cache and the expert's own keys/values (Eq. 1), followed by an
+ * output projection, a SwiGLU block and a waypoint head. One call = one tick.
+ *
+ * Conventions for every entry point:
+ *   - Pointers marked "device" must point to memory of the handle's device;
+ *     "host" pointers to ordinary (pageable or pinned) host memory.
+ *   - The caller owns every buffer it passes; the library never frees,
+ *     retains or writes any caller buffer except the documented outputs.
+ *   - Streams are passed as void* holding a cudaStream_t (NULL = legacy
+ *     default stream). Work is enqueued asynchronously unless stated.
+ *   - Every function returns an fsx_status; on failure a thread-local message
+ *     is available from fsx_last_error(). Host-side argument checks happen
+ *     before anything is enqueued.
+ *   - Supported shapes: head_dim == 128, d_model % 64 == 0, d_model <= 1024,
+ *     d_ff % 64 == 0, 1 <= n_action + n_frame <= 48, 1 <= n_waypoints <=
+ *     n_action + n_frame, n_layers <= 128. Other shapes give FSX_ERR_UNSUPPORTED.
+ *   - Precision: weights are stored as fp16 (round-to-nearest-even from the
+ *     fp32 host copy; exact for bf16-valued weights), GEMM and attention
+ *     operands are fp16 with fp32 accumulation, the residual stream, RMSNorm,
+ *     softmax statistics and the head are fp32. Cache values are converted to
+ *     fp16 on load and must lie within +-65504.
+ */
+#ifndef FSX_H
+#define FSX_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct fsx_handle_s* fsx_handle;
+
+typedef enum {
+  FSX_OK = 0,
+  FSX_ERR_INVALID_ARG = 1,  /* a host-checked argument is wrong                */
+  FSX_ERR_UNSUPPORTED = 2,  /* a shape or dtype outside the supported set      */
+  FSX_ERR_OOM = 3,          /* a device or host allocation failed              */
+  FSX_ERR_CUDA = 4,         /* a CUDA runtime call failed (see fsx_last_error) */
+  FSX_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up              */
+  FSX_ERR_DEVICE_ARG = 6    /* device-side check: offsets not non-decreasing,
+                               negative, or beyond max_total_cache_tokens      */
+} fsx_status;
+
+typedef enum { FSX_F32 = 0, FSX_BF16 = 1 } fsx_dtype;
+
+/* Model and capacity description, fixed at fsx_create. */
+typedef struct {
+  int n_layers;      /* expert layers == backbone layers (32); layer l reads cache layer l */
+  int d_model;       /* expert width d_ae (512)                                     */
+  int n_heads;       /* backbone attention heads (32)                               */
+  int head_dim;      /* backbone head width (128)                                   */
+  int d_ff;          /* SwiGLU hidden width (1408)                                  */
+  int n_action;      /* learned action tokens per vehicle (10)                      */
+  int n_frame;       /* frame tokens per vehicle (32)                               */
+  int n_waypoints;   /* waypoints per vehicle, read from action tokens 0.. (5)      */
+  int max_batch;     /* largest B any later fsx_tick may pass                       */
+  long long max_total_cache_tokens; /* largest offsets[B] any later tick may pass   */
+  int cache_dtype;   /* fsx_dtype of the K/V cache rows                             */
+  int frame_dtype;   /* fsx_dtype of the frame tokens                               */
+} fsx_config;
+
+/* Host fp32 expert weights, copied (and converted) by fsx_create; every matrix
+ * is row-major [out_features, in_features] and stacked over layers. */
+typedef struct {
+  const float* act_emb;    /* [n_action, d]                     learned action tokens  */
+  const float* pos_emb;    /* [n_action + n_frame, d]           learned positions      */
+  const float* attn_norm;  /* [n_layers, d]                     RMSNorm gain, attention*/
+  const float* wq;         /* [n_layers, n_heads*head_dim, d]   W_q (Sec. 3.1)         */
+  const float* wk;         /* [n_layers, n_heads*head_dim, d]   W_k                    */
+  const float* wv;         /* [n_layers, n_heads*head_dim, d]   W_v                    */
+  const float* wo;         /* [n_layers, d, n_heads*head_dim]   output projection      */
+  const float* mlp_norm;   /* [n_layers, d]                     RMSNorm gain, SwiGLU   */
+  const float* w_gate;     /* [n_layers, d_ff, d]               SwiGLU gate            */
+  const float* w_up;       /* [n_layers, d_ff, d]               SwiGLU up              */
+  const float* w_down;     /* [n_layers, d, d_ff]               SwiGLU down            */
+  const float* final_norm; /* [d]                               RMSNorm gain, head     */
+  const float* head_w;     /* [2, d]                            waypoint head          */
+  const float* head_b;     /* [2]                               waypoint head bias     */
+} fsx_weights;
+
+/* Create a handle on `device`: validates cfg (host), uploads fp16 weights in
+ * the kernels' tile order, allocates workspace for cfg->max_batch vehicles.
+ * Blocking. Errors: INVALID_ARG (null/negative fields), UNSUPPORTED (shape),
+ * OOM, CUDA. Env FSX_TEST_FAIL_ALLOC=1 forces the OOM path (tests). */
+fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, fsx_handle* out);
+
+/* One expert tick for B vehicles (Sec. 3.1, Eq. 1; Sec. 3.3: the cache is read
+ * as-is and never written).
+ *   k_cache, v_cache : HOST arrays of n_layers DEVICE pointers; layer l points
+ *                      to [total_tokens, n_heads, head_dim] rows of
+ *                      cfg.cache_dtype, token-major, vehicle b owning rows
+ *                      offsets[b] .. offsets[b+1]-1. Read only.
+ *   d_offsets        : DEVICE int64 [B+1], non-decreasing, offsets[0] >= 0,
+ *                      offsets[B] <= max_total_cache_tokens. L_b may be 0.
+ *   B                : 1 .. max_batch.
+ *   d_frames         : DEVICE [B, n_frame, d_model] of cfg.frame_dtype.
+ *   d_waypoints      : DEVICE fp32 [B, n_waypoints, 2] output.
+ * Enqueued on `stream` as one CUDA-graph launch (plus a small argument upload
+ * when any pointer changed since the previous tick); no host synchronisation.
+ * Device-side checks (offsets) set a sticky status read by fsx_get_status and
+ * turn the remaining kernels of the tick into no-ops. A handle must not run
+ * two ticks concurrently; ticks on different streams are serialised by the
+ * handle. Must not be called while `stream` is being captured. */
+fsx_status fsx_tick(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                    const int64_t* d_offsets, int B, const void* d_frames,
+                    float* d_waypoints, void* stream);
+
+/* fsx_tick with HOST frames, offsets and waypoints: copies h_offsets [B+1]
+ * and h_frames [B, n_frame, d] to handle-owned device buffers, runs the
+ * tick, copies the waypoints back to h_waypoints [B, n_waypoints, 2] and
+ * synchronises `stream`. The caches stay device-resident (k/v as in fsx_tick). */
+fsx_status fsx_tick_host(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                         const int64_t* h_offsets, int B, const void* h_frames,
+                         float* h_waypoints, void* stream);
+
+/* Same tick, launched kernel by kernel (no graph), additionally copying every
+ * layer's Eq. 1 output (before W_o) to d_attn_out: DEVICE fp16
+ * [n_layers, B*(n_action+n_frame), n_heads*head_dim]. For tests. */
+fsx_status fsx_tick_debug(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                          const int64_t* d_offsets, int B, const void* d_frames,
+                          float* d_waypoints, void* d_attn_out, void* stream);
+
+/* Synchronises `stream`, then returns and clears the device status word
+ * (FSX_OK, FSX_ERR_DEVICE_ARG or FSX_ERR_TIMEOUT). */
+fsx_status fsx_get_status(fsx_handle h, void* stream);
+
+/* Thread-local message describing the last failure on this thread ("" if none). */
+const char* fsx_last_error(void);
+
+/* Releases the handle's device memory and graphs (synchronises its device). */
+void fsx_destroy(fsx_handle h);
+
+/* Bytes of the handle's fp16 weight arena (algorithmic weight bytes per tick). */
+long long fsx_weight_bytes(fsx_handle h);
+
+/* Kernel launches one tick performs for batch B (what a graph replay runs). */
+int fsx_tick_launches(fsx_handle h, int B);
+
+/* Per-kernel-class timing of graph ticks, for roofline reports. With enable=1
+ * later fsx_tick calls replay a graph variant that records CUDA events around
+ * every launch of kernel class `kclass` (0 = QKV projection, 1 = attention,
+ * 2 = output projection, 3 = SwiGLU gate/up, 4 = down projection). fsx_kernel_time
+ * returns the summed event time (ms) and launch count of the most recent tick
+ * (synchronises the stream of that tick). */
+fsx_status fsx_set_kernel_timing(fsx_handle h, int enable, int kclass);
+fsx_status fsx_kernel_time(fsx_handle h, float* ms, int* launches);
+
+/* Eq. 1 alone (split-KV attention over [cache ; own], then the merge of the
+ * splits), for B vehicles and every head, fp16 in / fp16 out.
+ *   d_q      : DEVICE fp16, query row i of vehicle b at d_q + (b*n_q+i)*q_stride,
+ *              n_heads*head_dim wide (head h at column h*head_dim).
+ *   d_k_own, d_v_own : DEVICE fp16, own key/value row j of vehicle b at
+ *              + (b*n_own+j)*own_stride (same column layout).
+ *   d_k_cache, d_v_cache, d_offsets : as one layer of fsx_tick.
+ *   n_q in 1..48, n_own >= 0, n_splits in 1..64 (keys of vehicle b are cut
+ *   into n_splits near-equal ranges), head_dim == 128.
+ *   d_out    : DEVICE fp16 [B*n_q, n_heads*head_dim].
+ *   d_lse    : DEVICE fp32 [B, n_heads, n_q] natural-log log-sum-exp of the
+ *              scaled scores, or NULL.
+ *   d_workspace : DEVICE scratch of fsx_attention_workspace_bytes(...) bytes:
+ *              a status word, then the per-split partial outputs. Only this
+ *              call's kernels touch it; it must not be shared by calls that
+ *              overlap on the GPU. Asynchronous on `stream`; cache offsets
+ *              outside [0, ...] non-decreasing order make the kernels write
+ *              nothing. */
+size_t fsx_attention_workspace_bytes(int B, int n_heads, int n_q, int n_splits);
+fsx_status fsx_attention(const void* d_q, long long q_stride,
+                         const void* d_k_own, const void* d_v_own, long long own_stride,
+                         int n_q, int n_own,
+                         const void* d_k_cache, const void* d_v_cache, int cache_dtype,
+                         const int64_t* d_offsets, int B, int n_heads, int head_dim,
+                         int n_splits, void* d_out, float* d_lse,
+                         void* d_workspace, size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FSX_H */

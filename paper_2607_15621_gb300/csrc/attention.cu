@@ -1,0 +1,417 @@
+// Eq. 1 of Sec. 3.1: the expert's queries of one vehicle and one head attend,
+// with a single softmax, over the concatenation [K_vlm ; K_ae] / [V_vlm ; V_ae]
+// of that layer's backbone cache rows (read only) and the expert's own keys and
+// values. No mask, no rotary phase on the expert side, scale 1/sqrt(128).
+//
+// Split-KV flash decoding: the L_b + T keys of a vehicle are cut into
+// n_splits near-equal ranges; one CTA (3 warps x 16 queries = 48 query rows)
+// streams its range in 64-key chunks. Chunks are staged raw (bf16 / fp32 cache
+// rows, fp16 own rows) with 16-byte cp.async into a double buffer, converted
+// once to fp16 into an XOR-swizzled tile, and consumed by mma.sync m16n8k16
+// (S = Q K^T, then O += P V with P kept in registers) under an online softmax
+// in the log2 domain. With one split the CTA writes the normalised output;
+// otherwise it writes (O / l, m + log2 l) partials and a second kernel merges
+// them: lse = log2 sum_s 2^lse_s, o = sum_s 2^(lse_s - lse) o_s.
+#include <math_constants.h>
+
+#include "device_util.cuh"
+#include "kernels.h"
+
+namespace fsx {
+
+namespace {
+
+constexpr int kWarps = 3;
+constexpr int kThreads = kWarps * 32;
+constexpr int kChunk = 64;
+constexpr int kD = kHeadDim;           // 128
+constexpr int kUnits = kD * 2 / 16;    // 16-byte units per fp16 row (16)
+
+template <typename CT>
+struct CacheRow {
+  static constexpr int kBytes = kD * static_cast<int>(sizeof(CT));
+};
+
+// raw staging: [2 stages][K|V][kChunk rows][row bytes]; compute tiles: fp16 [K|V][kChunk][kD] swizzled
+template <typename CT>
+__host__ __device__ constexpr size_t attn_smem_bytes() {
+  return static_cast<size_t>(2) * 2 * kChunk * CacheRow<CT>::kBytes + static_cast<size_t>(2) * kChunk * kD * 2;
+}
+
+__device__ __forceinline__ int swz(int row, int unit) { return row * kUnits + (unit ^ (row & 7)); }
+
+template <typename CT>
+__device__ __forceinline__ void convert_unit(const unsigned char* raw, uint4* dst, bool own);
+
+// bf16 cache rows: 16 raw bytes = 8 values -> 8 fp16
+template <>
+__device__ __forceinline__ void convert_unit<__nv_bfloat16>(const unsigned char* raw, uint4* dst, bool own) {
+  const uint4 v = *reinterpret_cast<const uint4*>(raw);
+  if (own) {
+    *dst = v;
+  } else {
+    *dst = make_uint4(bf16x2_to_half2(v.x), bf16x2_to_half2(v.y), bf16x2_to_half2(v.z), bf16x2_to_half2(v.w));
+  }
+}
+
+// fp32 cache rows: 32 raw bytes = 8 values -> 8 fp16 (own rows are fp16 in the first half)
+template <>
+__device__ __forceinline__ void convert_unit<float>(const unsigned char* raw, uint4* dst, bool own) {
+  if (own) {
+    *dst = *reinterpret_cast<const uint4*>(raw);
+  } else {
+    const float4 a = *reinterpret_cast<const float4*>(raw);
+    const float4 b = *reinterpret_cast<const float4*>(raw + 16);
+    *dst = make_uint4(pack_half2(a.x, a.y), pack_half2(a.z, a.w), pack_half2(b.x, b.y), pack_half2(b.z, b.w));
+  }
+}
+
+template <typename CT>
+__global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  constexpr int RB = CacheRow<CT>::kBytes;
+  unsigned char* raw = smem;                                              // [2][2][kChunk][RB]
+  uint4* tile = reinterpret_cast<uint4*>(smem + static_cast<size_t>(2) * 2 * kChunk * RB);
+  uint4* kt = tile;                      // fp16 K chunk, swizzled
+  uint4* vt = tile + kChunk * kUnits;    // fp16 V chunk, swizzled
+
+  const int split = blockIdx.x;
+  const int h = blockIdx.y;
+  const int b = blockIdx.z;
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
+  const int H = p.n_heads;
+
+  pdl_launch_dependents();
+  pdl_wait();
+  if (*reinterpret_cast<volatile int*>(p.status) != 0) return;
+
+  const CT* kc;
+  const CT* vc;
+  const int64_t* offs;
+  if (p.targs != nullptr) {
+    kc = static_cast<const CT*>(p.targs->k_cache[p.layer]);
+    vc = static_cast<const CT*>(p.targs->v_cache[p.layer]);
+    offs = p.targs->offsets;
+  } else {
+    kc = static_cast<const CT*>(p.k_cache);
+    vc = static_cast<const CT*>(p.v_cache);
+    offs = p.offsets;
+  }
+  const long long o_lo = offs[b];
+  const long long o_hi = offs[b + 1];
+  if (o_lo < 0 || o_hi < o_lo || o_hi > p.max_total) {  // never read outside the caller's cache
+    set_status(p.status, kStatusDeviceArg);
+    return;
+  }
+  const long long L = o_hi - o_lo;
+  const long long n_keys = L + p.n_own;
+  const long long kbeg = n_keys * split / p.n_splits;
+  const long long kend = n_keys * (split + 1) / p.n_splits;
+
+  // output slots
+  const size_t part_base = (static_cast<size_t>(b) * H + h) * p.n_splits + split;  // partial index
+
+  if (kend <= kbeg) {  // an empty key range contributes nothing
+    if (p.n_splits > 1) {
+      for (int i = tid; i < kTokTile; i += kThreads) p.part_lse[part_base * kTokTile + i] = -CUDART_INF_F;
+      float* po = p.part_o + part_base * kTokTile * kD;
+      for (int i = tid; i < kTokTile * kD; i += kThreads) po[i] = 0.f;
+    } else {
+      for (int i = tid; i < p.n_q * kD; i += kThreads) {
+        const int qi = i / kD;
+        const int d = i % kD;
+        p.out[(static_cast<size_t>(b) * p.n_q + qi) * p.out_stride + h * kD + d] = __float2half_rn(0.f);
+      }
+      if (p.lse != nullptr)
+        for (int i = tid; i < p.n_q; i += kThreads) p.lse[(static_cast<size_t>(b) * H + h) * p.n_q + i] = -CUDART_INF_F;
+    }
+    return;
+  }
+
+  // ---- stage chunk c (keys kbeg + 64c ...) into raw stage s
+  auto issue_chunk = [&](int c, int s) {
+    const long long c0 = kbeg + static_cast<long long>(c) * kChunk;
+    const int rows = static_cast<int>(min(static_cast<long long>(kChunk), kend - c0));
+    constexpr int UPR = RB / 16;  // 16-byte units per raw row
+    unsigned char* kr = raw + (static_cast<size_t>(s) * 2 + 0) * kChunk * RB;
+    unsigned char* vr = raw + (static_cast<size_t>(s) * 2 + 1) * kChunk * RB;
+    for (int i = tid; i < rows * UPR; i += kThreads) {
+      const int r = i / UPR;
+      const int u = i - r * UPR;
+      const long long key = c0 + r;
+      const void* ks;
+      const void* vs;
+      if (key < L) {
+        const size_t row = (static_cast<size_t>(o_lo + key) * H + h) * kD;
+        ks = reinterpret_cast<const unsigned char*>(kc + row) + u * 16;
+        vs = reinterpret_cast<const unsigned char*>(vc + row) + u * 16;
+      } else {
+        if (u * 16 >= kD * 2) continue;  // own rows are fp16 (256 bytes)
+        const size_t row = (static_cast<size_t>(b) * p.n_own + static_cast<size_t>(key - L)) * p.own_stride + h * kD;
+        ks = reinterpret_cast<const unsigned char*>(p.k_own + row) + u * 16;
+        vs = reinterpret_cast<const unsigned char*>(p.v_own + row) + u * 16;
+      }
+      cp_async_16(smem_addr(kr + static_cast<size_t>(r) * RB + u * 16), ks);
+      cp_async_16(smem_addr(vr + static_cast<size_t>(r) * RB + u * 16), vs);
+    }
+    cp_async_commit();
+  };
+
+  // ---- Q fragments (A operand, 16 queries x 128) straight from global
+  const int qr0 = warp * 16 + (lane >> 2);
+  const int qr1 = qr0 + 8;
+  uint32_t qf[8][4];
+  {
+    const __half* q0 = p.q + (static_cast<size_t>(b) * p.n_q + qr0) * p.q_stride + h * kD;
+    const __half* q1 = p.q + (static_cast<size_t>(b) * p.n_q + qr1) * p.q_stride + h * kD;
+    const bool v0 = qr0 < p.n_q;
+    const bool v1 = qr1 < p.n_q;
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) {
+      const int c = kk * 16 + 2 * (lane & 3);
+      qf[kk][0] = v0 ? *reinterpret_cast<const uint32_t*>(q0 + c) : 0u;
+      qf[kk][1] = v1 ? *reinterpret_cast<const uint32_t*>(q1 + c) : 0u;
+      qf[kk][2] = v0 ? *reinterpret_cast<const uint32_t*>(q0 + c + 8) : 0u;
+      qf[kk][3] = v1 ? *reinterpret_cast<const uint32_t*>(q1 + c + 8) : 0u;
+    }
+  }
+
+  float o_acc[16][4];
+#pragma unroll
+  for (int n = 0; n < 16; ++n)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) o_acc[n][e] = 0.f;
+  float m_run[2] = {-CUDART_INF_F, -CUDART_INF_F};
+  float l_run[2] = {0.f, 0.f};
+  const float scale_log2 = 1.4426950408889634f * rsqrtf(static_cast<float>(kD));
+
+  const int n_chunks = static_cast<int>((kend - kbeg + kChunk - 1) / kChunk);
+  issue_chunk(0, 0);
+  if (n_chunks > 1) issue_chunk(1, 1);
+
+  for (int c = 0; c < n_chunks; ++c) {
+    const int s = c & 1;
+    if (c + 1 < n_chunks) cp_async_wait<1>(); else cp_async_wait<0>();
+    __syncthreads();  // raw stage s complete for everyone; previous tile consumers done
+
+    // ---- convert raw stage s -> fp16 swizzled tiles (rows beyond the range are zero)
+    const long long c0 = kbeg + static_cast<long long>(c) * kChunk;
+    const int rows = static_cast<int>(min(static_cast<long long>(kChunk), kend - c0));
+    {
+      const unsigned char* kr = raw + (static_cast<size_t>(s) * 2 + 0) * kChunk * RB;
+      const unsigned char* vr = raw + (static_cast<size_t>(s) * 2 + 1) * kChunk * RB;
+      constexpr int SRC_UNIT = RB / kUnits;  // raw bytes per 16-byte fp16 unit
+      for (int i = tid; i < kChunk * kUnits; i += kThreads) {
+        const int r = i / kUnits;
+        const int u = i - r * kUnits;
+        uint4* kd = kt + swz(r, u);
+        uint4* vd = vt + swz(r, u);
+        if (r < rows) {
+          const bool own = (c0 + r) >= L;
+          const int off = own ? u * 16 : u * SRC_UNIT;
+          convert_unit<CT>(kr + static_cast<size_t>(r) * RB + off, kd, own);
+          convert_unit<CT>(vr + static_cast<size_t>(r) * RB + off, vd, own);
+        } else {
+          *kd = make_uint4(0u, 0u, 0u, 0u);
+          *vd = make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+    }
+    __syncthreads();  // tiles ready, raw stage s free
+    if (c + 2 < n_chunks) issue_chunk(c + 2, s);
+
+    // ---- S = Q K^T for 16 queries x 64 keys
+    float sc[8][4];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) sc[j][e] = 0.f;
+#pragma unroll
+      for (int dd = 0; dd < 4; ++dd) {  // 32 dims per ldmatrix.x4
+        const int row = j * 8 + (lane & 7);
+        const int unit = dd * 4 + (lane >> 3);
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(b0, b1, b2, b3, smem_addr(kt + swz(row, unit)));
+        mma_f16_16816(sc[j], qf[2 * dd][0], qf[2 * dd][1], qf[2 * dd][2], qf[2 * dd][3], b0, b1);
+        mma_f16_16816(sc[j], qf[2 * dd + 1][0], qf[2 * dd + 1][1], qf[2 * dd + 1][2], qf[2 * dd + 1][3], b2, b3);
+      }
+    }
+    // ---- online softmax (log2 domain), masking keys past the range
+    float mx[2] = {-CUDART_INF_F, -CUDART_INF_F};
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int key = j * 8 + 2 * (lane & 3);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const bool valid = (key + (e & 1)) < rows;
+        sc[j][e] = valid ? sc[j][e] * scale_log2 : -CUDART_INF_F;
+      }
+      mx[0] = fmaxf(mx[0], fmaxf(sc[j][0], sc[j][1]));
+      mx[1] = fmaxf(mx[1], fmaxf(sc[j][2], sc[j][3]));
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
+      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
+    }
+    float alpha[2], m_new[2], rs[2] = {0.f, 0.f};
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      m_new[r] = fmaxf(m_run[r], mx[r]);
+      alpha[r] = exp2f(m_run[r] - m_new[r]);
+      m_run[r] = m_new[r];
+    }
+    uint32_t pf[4][4];  // P as A fragments, 4 k16 steps of 16 keys
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float p0 = exp2f(sc[j][0] - m_new[0]);
+      const float p1 = exp2f(sc[j][1] - m_new[0]);
+      const float p2 = exp2f(sc[j][2] - m_new[1]);
+      const float p3 = exp2f(sc[j][3] - m_new[1]);
+      rs[0] += p0 + p1;
+      rs[1] += p2 + p3;
+      const int kk = j >> 1;
+      if ((j & 1) == 0) {
+        pf[kk][0] = pack_half2(p0, p1);
+        pf[kk][1] = pack_half2(p2, p3);
+      } else {
+        pf[kk][2] = pack_half2(p0, p1);
+        pf[kk][3] = pack_half2(p2, p3);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      rs[r] += __shfl_xor_sync(0xffffffffu, rs[r], 1);
+      rs[r] += __shfl_xor_sync(0xffffffffu, rs[r], 2);
+      l_run[r] = l_run[r] * alpha[r] + rs[r];
+    }
+#pragma unroll
+    for (int n = 0; n < 16; ++n) {
+      o_acc[n][0] *= alpha[0];
+      o_acc[n][1] *= alpha[0];
+      o_acc[n][2] *= alpha[1];
+      o_acc[n][3] *= alpha[1];
+    }
+    // ---- O += P V
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+#pragma unroll
+      for (int np = 0; np < 8; ++np) {  // pairs of 8-wide d tiles
+        const int row = kk * 16 + (lane & 7) + 8 * ((lane >> 3) & 1);
+        const int unit = np * 2 + (lane >> 4);
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_trans(b0, b1, b2, b3, smem_addr(vt + swz(row, unit)));
+        mma_f16_16816(o_acc[2 * np], pf[kk][0], pf[kk][1], pf[kk][2], pf[kk][3], b0, b1);
+        mma_f16_16816(o_acc[2 * np + 1], pf[kk][0], pf[kk][1], pf[kk][2], pf[kk][3], b2, b3);
+      }
+    }
+  }
+
+  // ---- write out
+  const float inv0 = 1.f / l_run[0];
+  const float inv1 = 1.f / l_run[1];
+  if (p.n_splits == 1) {
+    const bool v0 = qr0 < p.n_q;
+    const bool v1 = qr1 < p.n_q;
+    __half* out0 = p.out + (static_cast<size_t>(b) * p.n_q + qr0) * p.out_stride + h * kD;
+    __half* out1 = p.out + (static_cast<size_t>(b) * p.n_q + qr1) * p.out_stride + h * kD;
+#pragma unroll
+    for (int n = 0; n < 16; ++n) {
+      const int d = n * 8 + 2 * (lane & 3);
+      if (v0) *reinterpret_cast<uint32_t*>(out0 + d) = pack_half2(o_acc[n][0] * inv0, o_acc[n][1] * inv0);
+      if (v1) *reinterpret_cast<uint32_t*>(out1 + d) = pack_half2(o_acc[n][2] * inv1, o_acc[n][3] * inv1);
+    }
+    if (p.lse != nullptr && (lane & 3) == 0) {
+      const float ln2 = 0.6931471805599453f;
+      if (v0) p.lse[(static_cast<size_t>(b) * H + h) * p.n_q + qr0] = (m_run[0] + log2f(l_run[0])) * ln2;
+      if (v1) p.lse[(static_cast<size_t>(b) * H + h) * p.n_q + qr1] = (m_run[1] + log2f(l_run[1])) * ln2;
+    }
+  } else {
+    float* po = p.part_o + part_base * kTokTile * kD;
+#pragma unroll
+    for (int n = 0; n < 16; ++n) {
+      const int d = n * 8 + 2 * (lane & 3);
+      *reinterpret_cast<float2*>(po + static_cast<size_t>(qr0) * kD + d) =
+          make_float2(o_acc[n][0] * inv0, o_acc[n][1] * inv0);
+      *reinterpret_cast<float2*>(po + static_cast<size_t>(qr1) * kD + d) =
+          make_float2(o_acc[n][2] * inv1, o_acc[n][3] * inv1);
+    }
+    if ((lane & 3) == 0) {
+      p.part_lse[part_base * kTokTile + qr0] = m_run[0] + log2f(l_run[0]);
+      p.part_lse[part_base * kTokTile + qr1] = m_run[1] + log2f(l_run[1]);
+    }
+  }
+}
+
+// Merge of the split partials of one (vehicle, head): 128 threads = 128 dims.
+__global__ void __launch_bounds__(kD) attn_combine_kernel(const AttnArgs p) {
+  const int h = blockIdx.x;
+  const int b = blockIdx.y;
+  const int d = threadIdx.x;
+  const int H = p.n_heads;
+  const int S = p.n_splits;
+  pdl_launch_dependents();
+  pdl_wait();
+  if (*reinterpret_cast<volatile int*>(p.status) != 0) return;
+  const size_t base = (static_cast<size_t>(b) * H + h) * S;
+  for (int qi = 0; qi < p.n_q; ++qi) {
+    float mmax = -CUDART_INF_F;
+    for (int s = 0; s < S; ++s) mmax = fmaxf(mmax, p.part_lse[(base + s) * kTokTile + qi]);
+    float wsum = 0.f;
+    float acc = 0.f;
+    if (mmax != -CUDART_INF_F) {
+      for (int s = 0; s < S; ++s) {
+        const float w = exp2f(p.part_lse[(base + s) * kTokTile + qi] - mmax);
+        wsum += w;
+        acc += w * p.part_o[((base + s) * kTokTile + qi) * kD + d];
+      }
+    }
+    const float o = wsum > 0.f ? acc / wsum : 0.f;
+    p.out[(static_cast<size_t>(b) * p.n_q + qi) * p.out_stride + h * kD + d] = __float2half_rn(o);
+    if (p.lse != nullptr && d == 0) {
+      p.lse[(static_cast<size_t>(b) * H + h) * p.n_q + qi] =
+          wsum > 0.f ? (mmax + log2f(wsum)) * 0.6931471805599453f : -CUDART_INF_F;
+    }
+  }
+}
+
+}  // namespace
+
+size_t attention_workspace_bytes(int B, int n_heads, int n_splits) {
+  if (n_splits <= 1) return 0;
+  const size_t parts = static_cast<size_t>(B) * n_heads * n_splits;
+  return parts * kTokTile * kD * sizeof(float) + parts * kTokTile * sizeof(float);
+}
+
+int attention_launch_count(int n_splits) { return n_splits > 1 ? 2 : 1; }
+
+cudaError_t attention_set_attributes() {
+  cudaError_t e = cudaFuncSetAttribute(reinterpret_cast<const void*>(&attn_splitkv_kernel<__nv_bfloat16>),
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(attn_smem_bytes<__nv_bfloat16>()));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(reinterpret_cast<const void*>(&attn_splitkv_kernel<float>),
+                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(attn_smem_bytes<float>()));
+}
+
+cudaError_t launch_attention(const AttnArgs& a_in, int B, int cache_dtype, cudaStream_t stream, bool pdl) {
+  AttnArgs a = a_in;
+  void* kargs[] = {&a};
+  const dim3 grid(a.n_splits, a.n_heads, B);
+  cudaError_t e;
+  if (cache_dtype == 1) {
+    e = launch_ex(reinterpret_cast<const void*>(&attn_splitkv_kernel<__nv_bfloat16>), grid, dim3(kThreads),
+                  attn_smem_bytes<__nv_bfloat16>(), stream, pdl, kargs);
+  } else {
+    e = launch_ex(reinterpret_cast<const void*>(&attn_splitkv_kernel<float>), grid, dim3(kThreads),
+                  attn_smem_bytes<float>(), stream, pdl, kargs);
+  }
+  if (e != cudaSuccess || a.n_splits <= 1) return e;
+  return launch_ex(reinterpret_cast<const void*>(&attn_combine_kernel), dim3(a.n_heads, B), dim3(kD), 0, stream,
+                   pdl, kargs);
+}
+
+}  // namespace fsx

@@ -1,0 +1,92 @@
+// Token assembly and waypoint head of the action expert (Sec. 3.1).
+//
+// embed: x_b = [E_act ; F_b] + P_pos into the fp32 residual stream; block 0
+//        also checks the cache offsets (non-decreasing, within capacity) and
+//        raises the device status word, which turns the rest of the tick
+//        into no-ops.
+// head:  waypoint j of vehicle b = W_h RMSNorm(x_{b,j}; g_f) + b_h, fp32.
+#include "device_util.cuh"
+#include "kernels.h"
+
+namespace fsx {
+
+namespace {
+
+__global__ void embed_kernel(const EmbedArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int T = a.n_action + a.n_frame;
+  const int row = blockIdx.x;  // b * T + t
+  const int b = row / T;
+  const int t = row - b * T;
+  if (row == 0 && threadIdx.x == 0) {
+    const int64_t* off = a.targs->offsets;
+    bool ok = off[0] >= 0;
+    for (int i = 0; i < a.B && ok; ++i) ok = off[i + 1] >= off[i];
+    ok = ok && off[a.B] <= a.max_total;
+    if (!ok) set_status(a.status, kStatusDeviceArg);
+  }
+  float* xr = a.x + static_cast<size_t>(row) * a.d;
+  const float* pos = a.pos_emb + static_cast<size_t>(t) * a.d;
+  for (int c = threadIdx.x; c < a.d; c += blockDim.x) {
+    float v;
+    if (t < a.n_action) {
+      v = a.act_emb[static_cast<size_t>(t) * a.d + c];
+    } else {
+      const size_t idx = (static_cast<size_t>(b) * a.n_frame + (t - a.n_action)) * a.d + c;
+      if (a.frame_dtype == 1) {
+        v = __bfloat162float(static_cast<const __nv_bfloat16*>(a.targs->frames)[idx]);
+      } else {
+        v = static_cast<const float*>(a.targs->frames)[idx];
+      }
+    }
+    xr[c] = v + pos[c];
+  }
+}
+
+// one warp per (vehicle, waypoint)
+__global__ void head_kernel(const HeadArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
+  if (*reinterpret_cast<volatile int*>(a.status) != 0) return;
+  const int b = blockIdx.x;
+  const int lane = threadIdx.x & 31;
+  for (int j = threadIdx.x >> 5; j < a.n_waypoints; j += blockDim.x >> 5) {
+  const float* xr = a.x + (static_cast<size_t>(b) * a.T + j) * a.d;
+  float ss = 0.f;
+  for (int c = lane; c < a.d; c += 32) ss += xr[c] * xr[c];
+  ss = warp_sum(ss);
+  const float rstd = rsqrtf(ss / static_cast<float>(a.d) + 1e-6f);
+  float o0 = 0.f, o1 = 0.f;
+  for (int c = lane; c < a.d; c += 32) {
+    const float n = xr[c] * rstd * a.final_norm[c];
+    o0 += a.head_w[c] * n;
+    o1 += a.head_w[a.d + c] * n;
+  }
+  o0 = warp_sum(o0);
+  o1 = warp_sum(o1);
+  if (lane == 0) {
+    float* out = a.targs != nullptr ? a.targs->waypoints : a.out;
+    out[(static_cast<size_t>(b) * a.n_waypoints + j) * 2 + 0] = o0 + a.head_b[0];
+    out[(static_cast<size_t>(b) * a.n_waypoints + j) * 2 + 1] = o1 + a.head_b[1];
+  }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_embed(const EmbedArgs& a_in, cudaStream_t stream, bool pdl) {
+  EmbedArgs a = a_in;
+  void* kargs[] = {&a};
+  const int rows = a.B * (a.n_action + a.n_frame);
+  return launch_ex(reinterpret_cast<const void*>(&embed_kernel), dim3(rows), dim3(128), 0, stream, pdl, kargs);
+}
+
+cudaError_t launch_head(const HeadArgs& a_in, cudaStream_t stream, bool pdl) {
+  HeadArgs a = a_in;
+  void* kargs[] = {&a};
+  return launch_ex(reinterpret_cast<const void*>(&head_kernel), dim3(a.B), dim3(32 * (a.n_waypoints < 8 ? a.n_waypoints : 8)), 0, stream,
+                   pdl, kargs);
+}
+
+}  // namespace fsx

@@ -1,0 +1,695 @@
+// C ABI of the action-expert tick (include/fsx.h): handle creation with fp16
+// weight packing, the per-tick launch sequence, CUDA-graph capture and replay,
+// the device status word and the test/measurement entry points.
+//
+// Per tick (Sec. 3.1; the expert runs at every tick of Sec. 3.3 and reads the
+// cache as-is):   embed -> 32 x [ RMSNorm+QKV -> Eq. 1 attention (+ merge)
+//                 -> W_o + residual -> RMSNorm+gate/up+SiLU -> W_d + residual ]
+//                 -> RMSNorm + waypoint head.
+// Every launch uses programmatic dependent launch, so each kernel can fetch
+// its weights while its predecessor finishes; the sequence for one batch size
+// is captured once into a CUDA graph and replayed by every later tick.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <thread>
+#include <vector>
+
+#include "../../include/fsx.h"
+#include "kernels.h"
+
+using fsx::TickArgs;
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+fsx_status fail(fsx_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+#define FSX_CUDA(call)                                                                              \
+  do {                                                                                              \
+    cudaError_t e_ = (call);                                                                        \
+    if (e_ != cudaSuccess) return fail(FSX_ERR_CUDA, "%s: %s (%s:%d)", #call, cudaGetErrorString(e_), \
+                                       __FILE__, __LINE__);                                         \
+  } while (0)
+
+constexpr int kClassQkv = 0, kClassAttn = 1, kClassWo = 2, kClassGateUp = 3, kClassDown = 4;
+
+}  // namespace
+
+struct fsx_handle_s {
+  fsx_config cfg{};
+  int device = 0;
+  int sm_count = 0;
+  int T = 0;
+  int HD = 0;
+  // packed fp16 weights
+  void* w_arena = nullptr;
+  long long weight_bytes = 0;
+  std::vector<const uint4*> w_qkv, w_o, w_gu, w_dn;
+  // fp32 small parameters
+  float* params = nullptr;
+  float *act_emb = nullptr, *pos_emb = nullptr, *attn_norm = nullptr, *mlp_norm = nullptr;
+  float *final_norm = nullptr, *head_w = nullptr, *head_b = nullptr;
+  // workspace
+  float* x = nullptr;
+  __half* qkv = nullptr;
+  __half* o = nullptr;
+  __half* hbuf = nullptr;
+  float* part = nullptr;
+  size_t part_bytes = 0;
+  int* status = nullptr;
+  TickArgs* d_args = nullptr;
+  TickArgs h_args{};
+  bool args_valid = false;
+  // host-buffer tick staging
+  int64_t* st_offsets = nullptr;
+  void* st_frames = nullptr;
+  float* st_waypoints = nullptr;
+  // graphs
+  cudaStream_t cap_stream = nullptr;
+  std::map<int, cudaGraphExec_t> graphs;
+  std::map<int, cudaGraphExec_t> timed_graphs;
+  bool timing = false;
+  int timing_class = 0;
+  std::vector<cudaEvent_t> tev;
+  int timed_pairs = 0;
+  bool timed_pending = false;
+  cudaEvent_t last_tick = nullptr;
+  cudaStream_t last_stream = nullptr;
+  bool has_last = false;
+  std::mutex mu;
+};
+
+namespace {
+
+int attention_splits(const fsx_handle_s* h, int B) {
+  const int work = B * h->cfg.n_heads;
+  int s = (2 * h->sm_count) / std::max(work, 1);
+  return std::min(std::max(s, 1), 16);
+}
+
+fsx_status check_config(const fsx_config* c) {
+  if (!c) return fail(FSX_ERR_INVALID_ARG, "config is NULL");
+  if (c->n_layers <= 0 || c->d_model <= 0 || c->n_heads <= 0 || c->head_dim <= 0 || c->d_ff <= 0 ||
+      c->n_action <= 0 || c->n_frame < 0 || c->n_waypoints <= 0 || c->max_batch <= 0 ||
+      c->max_total_cache_tokens < 0)
+    return fail(FSX_ERR_INVALID_ARG, "config fields must be positive (n_frame, max_total_cache_tokens >= 0)");
+  if ((c->cache_dtype != FSX_F32 && c->cache_dtype != FSX_BF16) ||
+      (c->frame_dtype != FSX_F32 && c->frame_dtype != FSX_BF16))
+    return fail(FSX_ERR_INVALID_ARG, "cache_dtype / frame_dtype must be FSX_F32 or FSX_BF16");
+  const int T = c->n_action + c->n_frame;
+  if (c->n_waypoints > T) return fail(FSX_ERR_INVALID_ARG, "n_waypoints exceeds the token count");
+  if (c->head_dim != fsx::kHeadDim) return fail(FSX_ERR_UNSUPPORTED, "head_dim must be 128");
+  if (c->d_model % 64 != 0 || c->d_model > 1024) return fail(FSX_ERR_UNSUPPORTED, "d_model must be a multiple of 64, <= 1024");
+  if (c->d_ff % 64 != 0) return fail(FSX_ERR_UNSUPPORTED, "d_ff must be a multiple of 64");
+  if (T > fsx::kTokTile) return fail(FSX_ERR_UNSUPPORTED, "n_action + n_frame must be <= 48");
+  if (c->n_layers > fsx::kMaxLayers) return fail(FSX_ERR_UNSUPPORTED, "n_layers must be <= 128");
+  if (c->n_heads > 4096) return fail(FSX_ERR_UNSUPPORTED, "n_heads too large");
+  return FSX_OK;
+}
+
+// fp32 -> fp16 fragment blocks of the tensor-core A operand (m16n8k16):
+// block (nb, kb) holds, for lane l, rows r = 16nb + l/4 and r + 8 and columns
+// c = 16kb + 2(l%4) (+1, +8, +9) in register order a0..a7.
+template <typename RowFn>
+void pack_fragments(RowFn row, int N, int K, __half* out) {
+  const int kbs = K / 16;
+  for (int nb = 0; nb < N / 16; ++nb) {
+    for (int lane = 0; lane < 32; ++lane) {
+      const float* r0 = row(nb * 16 + (lane >> 2));
+      const float* r1 = row(nb * 16 + (lane >> 2) + 8);
+      const int c = 2 * (lane & 3);
+      for (int kb = 0; kb < kbs; ++kb) {
+        __half* o = out + ((static_cast<size_t>(nb) * kbs + kb) * 32 + lane) * 8;
+        const int k = kb * 16 + c;
+        o[0] = __float2half_rn(r0[k]);
+        o[1] = __float2half_rn(r0[k + 1]);
+        o[2] = __float2half_rn(r1[k]);
+        o[3] = __float2half_rn(r1[k + 1]);
+        o[4] = __float2half_rn(r0[k + 8]);
+        o[5] = __float2half_rn(r0[k + 9]);
+        o[6] = __float2half_rn(r1[k + 8]);
+        o[7] = __float2half_rn(r1[k + 9]);
+      }
+    }
+  }
+}
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_capture, bool timed) {
+  const fsx_config& c = h->cfg;
+  const int d = c.d_model, HD = h->HD, F = c.d_ff, T = h->T;
+  const int M = B * T;
+  const bool pdl = true;
+  int pair = 0;
+  auto mark = [&](int cls, bool begin) -> cudaError_t {
+    if (!timed || cls != h->timing_class) return cudaSuccess;
+    cudaEvent_t ev = h->tev[2 * pair + (begin ? 0 : 1)];
+    if (!begin) ++pair;
+    return cudaEventRecordWithFlags(ev, st, cudaEventRecordExternal);
+  };
+
+  fsx::EmbedArgs ea{};
+  ea.act_emb = h->act_emb;
+  ea.pos_emb = h->pos_emb;
+  ea.targs = h->d_args;
+  ea.frame_dtype = c.frame_dtype;
+  ea.n_action = c.n_action;
+  ea.n_frame = c.n_frame;
+  ea.d = d;
+  ea.B = B;
+  ea.max_total = c.max_total_cache_tokens;
+  ea.x = h->x;
+  ea.status = h->status;
+  FSX_CUDA(fsx::launch_embed(ea, st, pdl));
+
+  const fsx::GemmPlan pq = fsx::plan_gemm(3 * HD, d, M, 2, d, fsx::kProNorm, fsx::kEpiStore, h->sm_count);
+  const fsx::GemmPlan po = fsx::plan_gemm(d, HD, M, 2, 512, fsx::kProCopy, fsx::kEpiAtomic, h->sm_count);
+  const fsx::GemmPlan pg = fsx::plan_gemm(2 * F, d, M, 1, d, fsx::kProNorm, fsx::kEpiSwiglu, h->sm_count);
+  const fsx::GemmPlan pd = fsx::plan_gemm(d, F, M, 1, 256, fsx::kProCopy, fsx::kEpiAtomic, h->sm_count);
+  const int S = attention_splits(h, B);
+
+  for (int l = 0; l < c.n_layers; ++l) {
+    fsx::GemmArgs g{};
+    g.M = M;
+    g.status = h->status;
+    // RMSNorm + [W_q; W_k; W_v]
+    g.w = h->w_qkv[l];
+    g.n_rows = 3 * HD;
+    g.K = d;
+    g.x = h->x;
+    g.gamma = h->attn_norm + static_cast<size_t>(l) * d;
+    g.ldx = d;
+    g.y = h->qkv;
+    g.ldy = 3 * HD;
+    FSX_CUDA(mark(kClassQkv, true));
+    FSX_CUDA(fsx::launch_gemm(pq, g, st, pdl));
+    FSX_CUDA(mark(kClassQkv, false));
+
+    // Eq. 1 over [cache_l ; own]
+    fsx::AttnArgs a{};
+    a.q = h->qkv;
+    a.q_stride = 3 * HD;
+    a.k_own = h->qkv + HD;
+    a.v_own = h->qkv + 2 * HD;
+    a.own_stride = 3 * HD;
+    a.n_q = T;
+    a.n_own = T;
+    a.targs = h->d_args;
+    a.layer = l;
+    a.max_total = c.max_total_cache_tokens;
+    a.n_heads = c.n_heads;
+    a.n_splits = S;
+    a.out = h->o;
+    a.out_stride = HD;
+    a.lse = nullptr;
+    a.part_o = h->part;
+    a.part_lse = h->part + static_cast<size_t>(B) * c.n_heads * S * fsx::kTokTile * fsx::kHeadDim;
+    a.status = h->status;
+    FSX_CUDA(mark(kClassAttn, true));
+    FSX_CUDA(fsx::launch_attention(a, B, c.cache_dtype, st, pdl));
+    FSX_CUDA(mark(kClassAttn, false));
+    if (attn_capture) {
+      FSX_CUDA(cudaMemcpyAsync(attn_capture + static_cast<size_t>(l) * M * HD, h->o,
+                               static_cast<size_t>(M) * HD * sizeof(__half), cudaMemcpyDeviceToDevice, st));
+    }
+
+    // x += o W_o^T
+    fsx::GemmArgs go{};
+    go.M = M;
+    go.status = h->status;
+    go.w = h->w_o[l];
+    go.n_rows = d;
+    go.K = HD;
+    go.a = h->o;
+    go.lda = HD;
+    go.xo = h->x;
+    go.ldxo = d;
+    FSX_CUDA(mark(kClassWo, true));
+    FSX_CUDA(fsx::launch_gemm(po, go, st, pdl));
+    FSX_CUDA(mark(kClassWo, false));
+
+    // h = silu(RMSNorm(x) W_g^T) * (RMSNorm(x) W_u^T)
+    fsx::GemmArgs gg{};
+    gg.M = M;
+    gg.status = h->status;
+    gg.w = h->w_gu[l];
+    gg.n_rows = 2 * F;
+    gg.K = d;
+    gg.x = h->x;
+    gg.gamma = h->mlp_norm + static_cast<size_t>(l) * d;
+    gg.ldx = d;
+    gg.y = h->hbuf;
+    gg.ldy = F;
+    FSX_CUDA(mark(kClassGateUp, true));
+    FSX_CUDA(fsx::launch_gemm(pg, gg, st, pdl));
+    FSX_CUDA(mark(kClassGateUp, false));
+
+    // x += h W_d^T
+    fsx::GemmArgs gd{};
+    gd.M = M;
+    gd.status = h->status;
+    gd.w = h->w_dn[l];
+    gd.n_rows = d;
+    gd.K = F;
+    gd.a = h->hbuf;
+    gd.lda = F;
+    gd.xo = h->x;
+    gd.ldxo = d;
+    FSX_CUDA(mark(kClassDown, true));
+    FSX_CUDA(fsx::launch_gemm(pd, gd, st, pdl));
+    FSX_CUDA(mark(kClassDown, false));
+  }
+
+  fsx::HeadArgs ha{};
+  ha.x = h->x;
+  ha.final_norm = h->final_norm;
+  ha.head_w = h->head_w;
+  ha.head_b = h->head_b;
+  ha.targs = h->d_args;
+  ha.out = nullptr;
+  ha.d = d;
+  ha.T = T;
+  ha.n_waypoints = c.n_waypoints;
+  ha.B = B;
+  ha.status = h->status;
+  FSX_CUDA(fsx::launch_head(ha, st, pdl));
+  if (timed) h->timed_pairs = pair;
+  return FSX_OK;
+}
+
+fsx_status get_graph(fsx_handle_s* h, int B, bool timed, cudaGraphExec_t* out) {
+  auto& map = timed ? h->timed_graphs : h->graphs;
+  auto it = map.find(B);
+  if (it != map.end()) {
+    *out = it->second;
+    return FSX_OK;
+  }
+  FSX_CUDA(cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal));
+  fsx_status s = enqueue_tick(h, B, h->cap_stream, nullptr, timed);
+  cudaGraph_t graph = nullptr;
+  cudaError_t e = cudaStreamEndCapture(h->cap_stream, &graph);
+  if (s != FSX_OK) {
+    if (graph) cudaGraphDestroy(graph);
+    return s;
+  }
+  if (e != cudaSuccess) return fail(FSX_ERR_CUDA, "graph capture failed: %s", cudaGetErrorString(e));
+  cudaGraphExec_t exec = nullptr;
+  e = cudaGraphInstantiate(&exec, graph, 0);
+  cudaGraphDestroy(graph);
+  if (e != cudaSuccess) return fail(FSX_ERR_CUDA, "graph instantiate failed: %s", cudaGetErrorString(e));
+  map[B] = exec;
+  *out = exec;
+  return FSX_OK;
+}
+
+fsx_status check_tick_args(fsx_handle_s* h, const void* const* k_cache, const void* const* v_cache,
+                           const void* offsets, int B, const void* frames, const void* waypoints) {
+  if (!h) return fail(FSX_ERR_INVALID_ARG, "handle is NULL");
+  if (B < 1 || B > h->cfg.max_batch) return fail(FSX_ERR_INVALID_ARG, "B=%d outside 1..max_batch=%d", B, h->cfg.max_batch);
+  if (!k_cache || !v_cache) return fail(FSX_ERR_INVALID_ARG, "k_cache / v_cache pointer arrays are NULL");
+  for (int l = 0; l < h->cfg.n_layers; ++l)
+    if (!k_cache[l] || !v_cache[l]) return fail(FSX_ERR_INVALID_ARG, "cache pointer of layer %d is NULL", l);
+  if (!offsets) return fail(FSX_ERR_INVALID_ARG, "offsets is NULL");
+  if (!frames) return fail(FSX_ERR_INVALID_ARG, "frames is NULL");
+  if (!waypoints) return fail(FSX_ERR_INVALID_ARG, "waypoints is NULL");
+  return FSX_OK;
+}
+
+// Upload the per-tick pointers when they changed and order this tick after the
+// previous one if it was issued on another stream.
+fsx_status prepare_tick(fsx_handle_s* h, const void* const* k_cache, const void* const* v_cache,
+                        const int64_t* d_offsets, const void* d_frames, float* d_waypoints, cudaStream_t st) {
+  FSX_CUDA(cudaSetDevice(h->device));
+  if (h->has_last && h->last_stream != st) FSX_CUDA(cudaStreamWaitEvent(st, h->last_tick, 0));
+  TickArgs a{};
+  for (int l = 0; l < h->cfg.n_layers; ++l) {
+    a.k_cache[l] = k_cache[l];
+    a.v_cache[l] = v_cache[l];
+  }
+  a.offsets = d_offsets;
+  a.frames = d_frames;
+  a.waypoints = d_waypoints;
+  if (!h->args_valid || std::memcmp(&a, &h->h_args, sizeof(TickArgs)) != 0) {
+    h->h_args = a;
+    FSX_CUDA(cudaMemcpyAsync(h->d_args, &h->h_args, sizeof(TickArgs), cudaMemcpyHostToDevice, st));
+    h->args_valid = true;
+  }
+  return FSX_OK;
+}
+
+fsx_status finish_tick(fsx_handle_s* h, cudaStream_t st) {
+  FSX_CUDA(cudaEventRecord(h->last_tick, st));
+  h->last_stream = st;
+  h->has_last = true;
+  return FSX_OK;
+}
+
+void free_handle(fsx_handle_s* h) {
+  if (!h) return;
+  cudaSetDevice(h->device);
+  cudaDeviceSynchronize();
+  for (auto& kv : h->graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : h->timed_graphs) cudaGraphExecDestroy(kv.second);
+  for (cudaEvent_t e : h->tev) cudaEventDestroy(e);
+  if (h->last_tick) cudaEventDestroy(h->last_tick);
+  if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
+  void* bufs[] = {h->w_arena, h->params, h->x, h->qkv, h->o, h->hbuf, h->part, h->status, h->d_args,
+                  h->st_offsets, h->st_frames, h->st_waypoints};
+  for (void* p : bufs)
+    if (p) cudaFree(p);
+  delete h;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* fsx_last_error(void) { return g_err; }
+
+fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, fsx_handle* out) {
+  g_err[0] = '\0';
+  if (!out) return fail(FSX_ERR_INVALID_ARG, "out handle pointer is NULL");
+  *out = nullptr;
+  fsx_status s = check_config(cfg);
+  if (s != FSX_OK) return s;
+  if (!w || !w->act_emb || !w->pos_emb || !w->attn_norm || !w->wq || !w->wk || !w->wv || !w->wo ||
+      !w->mlp_norm || !w->w_gate || !w->w_up || !w->w_down || !w->final_norm || !w->head_w || !w->head_b)
+    return fail(FSX_ERR_INVALID_ARG, "a weight pointer is NULL");
+  if (device < 0) return fail(FSX_ERR_INVALID_ARG, "device must be >= 0");
+  const char* fa = std::getenv("FSX_TEST_FAIL_ALLOC");
+  if (fa && fa[0] == '1') return fail(FSX_ERR_OOM, "allocation failure forced by FSX_TEST_FAIL_ALLOC");
+
+  int n_dev = 0;
+  if (cudaGetDeviceCount(&n_dev) != cudaSuccess || n_dev == 0) return fail(FSX_ERR_CUDA, "no CUDA device available");
+  if (device >= n_dev) return fail(FSX_ERR_INVALID_ARG, "device %d >= device count %d", device, n_dev);
+
+  fsx_handle_s* h = new fsx_handle_s();
+  h->cfg = *cfg;
+  h->device = device;
+  h->T = cfg->n_action + cfg->n_frame;
+  h->HD = cfg->n_heads * cfg->head_dim;
+  const int L = cfg->n_layers, d = cfg->d_model, HD = h->HD, F = cfg->d_ff, T = h->T;
+
+  auto bail = [&](fsx_status st) {
+    free_handle(h);
+    return st;
+  };
+#define FSX_CUDA_H(call)                                                                                  \
+  do {                                                                                                    \
+    cudaError_t e_ = (call);                                                                              \
+    if (e_ != cudaSuccess)                                                                                \
+      return bail(fail(e_ == cudaErrorMemoryAllocation ? FSX_ERR_OOM : FSX_ERR_CUDA, "%s: %s", #call,    \
+                       cudaGetErrorString(e_)));                                                          \
+  } while (0)
+
+  FSX_CUDA_H(cudaSetDevice(device));
+  FSX_CUDA_H(cudaDeviceGetAttribute(&h->sm_count, cudaDevAttrMultiProcessorCount, device));
+  FSX_CUDA_H(fsx::gemm_set_attributes());
+  FSX_CUDA_H(fsx::attention_set_attributes());
+
+  // ---- packed fp16 weights: per layer [qkv | o | gate/up | down], 256-byte aligned
+  const size_t n_qkv = static_cast<size_t>(3) * HD * d, n_o = static_cast<size_t>(d) * HD;
+  const size_t n_gu = static_cast<size_t>(2) * F * d, n_dn = static_cast<size_t>(d) * F;
+  const size_t b_qkv = align_up(n_qkv * 2, 256), b_o = align_up(n_o * 2, 256);
+  const size_t b_gu = align_up(n_gu * 2, 256), b_dn = align_up(n_dn * 2, 256);
+  const size_t per_layer = b_qkv + b_o + b_gu + b_dn;
+  const size_t arena = per_layer * L;
+  h->weight_bytes = static_cast<long long>((n_qkv + n_o + n_gu + n_dn) * 2 * L);
+  FSX_CUDA_H(cudaMalloc(&h->w_arena, arena));
+  {
+    std::vector<__half> host(arena / 2);
+    const size_t hd_d = static_cast<size_t>(HD) * d;
+    auto pack_layer = [&](int l) {
+      unsigned char* base = reinterpret_cast<unsigned char*>(host.data()) + per_layer * l;
+      const float* wq = w->wq + hd_d * l;
+      const float* wk = w->wk + hd_d * l;
+      const float* wv = w->wv + hd_d * l;
+      pack_fragments(
+          [&](int r) -> const float* {
+            if (r < HD) return wq + static_cast<size_t>(r) * d;
+            if (r < 2 * HD) return wk + static_cast<size_t>(r - HD) * d;
+            return wv + static_cast<size_t>(r - 2 * HD) * d;
+          },
+          3 * HD, d, reinterpret_cast<__half*>(base));
+      const float* wo = w->wo + hd_d * l;
+      pack_fragments([&](int r) -> const float* { return wo + static_cast<size_t>(r) * HD; }, d, HD,
+                     reinterpret_cast<__half*>(base + b_qkv));
+      const float* wg = w->w_gate + static_cast<size_t>(F) * d * l;
+      const float* wu = w->w_up + static_cast<size_t>(F) * d * l;
+      // packed row p: block p/16, rows 0..7 gate rows 8*(p/16)+r, rows 8..15 the matching up rows
+      pack_fragments(
+          [&](int p) -> const float* {
+            const int blk = p >> 4, r = p & 15;
+            return r < 8 ? wg + static_cast<size_t>(blk * 8 + r) * d : wu + static_cast<size_t>(blk * 8 + r - 8) * d;
+          },
+          2 * F, d, reinterpret_cast<__half*>(base + b_qkv + b_o));
+      const float* wd = w->w_down + static_cast<size_t>(d) * F * l;
+      pack_fragments([&](int r) -> const float* { return wd + static_cast<size_t>(r) * F; }, d, F,
+                     reinterpret_cast<__half*>(base + b_qkv + b_o + b_gu));
+    };
+    const int n_threads = std::max(1, std::min<int>(16, static_cast<int>(std::thread::hardware_concurrency())));
+    std::vector<std::thread> pool;
+    for (int t = 0; t < n_threads; ++t)
+      pool.emplace_back([&, t]() {
+        for (int l = t; l < L; l += n_threads) pack_layer(l);
+      });
+    for (auto& th : pool) th.join();
+    FSX_CUDA_H(cudaMemcpy(h->w_arena, host.data(), arena, cudaMemcpyHostToDevice));
+  }
+  for (int l = 0; l < L; ++l) {
+    const unsigned char* base = static_cast<const unsigned char*>(h->w_arena) + per_layer * l;
+    h->w_qkv.push_back(reinterpret_cast<const uint4*>(base));
+    h->w_o.push_back(reinterpret_cast<const uint4*>(base + b_qkv));
+    h->w_gu.push_back(reinterpret_cast<const uint4*>(base + b_qkv + b_o));
+    h->w_dn.push_back(reinterpret_cast<const uint4*>(base + b_qkv + b_o + b_gu));
+  }
+
+  // ---- fp32 parameters
+  {
+    const size_t n_act = static_cast<size_t>(cfg->n_action) * d, n_pos = static_cast<size_t>(T) * d;
+    const size_t n_norm = static_cast<size_t>(L) * d;
+    std::vector<size_t> sizes = {n_act, n_pos, n_norm, n_norm, static_cast<size_t>(d), static_cast<size_t>(2) * d, 2};
+    std::vector<const float*> srcs = {w->act_emb, w->pos_emb, w->attn_norm, w->mlp_norm, w->final_norm, w->head_w, w->head_b};
+    size_t total = 0;
+    std::vector<size_t> offs;
+    for (size_t sz : sizes) {
+      offs.push_back(total);
+      total += align_up(sz, 64);
+    }
+    FSX_CUDA_H(cudaMalloc(&h->params, total * sizeof(float)));
+    for (size_t i = 0; i < sizes.size(); ++i)
+      FSX_CUDA_H(cudaMemcpy(h->params + offs[i], srcs[i], sizes[i] * sizeof(float), cudaMemcpyHostToDevice));
+    h->act_emb = h->params + offs[0];
+    h->pos_emb = h->params + offs[1];
+    h->attn_norm = h->params + offs[2];
+    h->mlp_norm = h->params + offs[3];
+    h->final_norm = h->params + offs[4];
+    h->head_w = h->params + offs[5];
+    h->head_b = h->params + offs[6];
+  }
+
+  // ---- workspace for max_batch
+  const size_t Mmax = static_cast<size_t>(cfg->max_batch) * T;
+  const size_t m_pad = (Mmax + fsx::kTokTile - 1) / fsx::kTokTile * fsx::kTokTile;
+  FSX_CUDA_H(cudaMalloc(&h->x, m_pad * d * sizeof(float)));
+  FSX_CUDA_H(cudaMalloc(&h->qkv, m_pad * 3 * HD * sizeof(__half)));
+  FSX_CUDA_H(cudaMalloc(&h->o, m_pad * HD * sizeof(__half)));
+  FSX_CUDA_H(cudaMalloc(&h->hbuf, m_pad * F * sizeof(__half)));
+  size_t part = 0;
+  for (int B = 1; B <= cfg->max_batch; ++B)
+    part = std::max(part, fsx::attention_workspace_bytes(B, cfg->n_heads, attention_splits(h, B)));
+  h->part_bytes = part;
+  if (part) FSX_CUDA_H(cudaMalloc(&h->part, part));
+  FSX_CUDA_H(cudaMalloc(&h->status, sizeof(int)));
+  FSX_CUDA_H(cudaMemset(h->status, 0, sizeof(int)));
+  FSX_CUDA_H(cudaMalloc(&h->d_args, sizeof(TickArgs)));
+  FSX_CUDA_H(cudaMalloc(&h->st_offsets, (cfg->max_batch + 1) * sizeof(int64_t)));
+  FSX_CUDA_H(cudaMalloc(&h->st_frames, static_cast<size_t>(cfg->max_batch) * cfg->n_frame * d * sizeof(float) + 16));
+  FSX_CUDA_H(cudaMalloc(&h->st_waypoints, static_cast<size_t>(cfg->max_batch) * cfg->n_waypoints * 2 * sizeof(float)));
+  FSX_CUDA_H(cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking));
+  FSX_CUDA_H(cudaEventCreateWithFlags(&h->last_tick, cudaEventDisableTiming));
+  h->tev.resize(2 * static_cast<size_t>(L));
+  for (auto& e : h->tev) FSX_CUDA_H(cudaEventCreate(&e));
+  FSX_CUDA_H(cudaDeviceSynchronize());
+#undef FSX_CUDA_H
+  *out = h;
+  return FSX_OK;
+}
+
+fsx_status fsx_tick(fsx_handle h, const void* const* k_cache, const void* const* v_cache, const int64_t* d_offsets,
+                    int B, const void* d_frames, float* d_waypoints, void* stream) {
+  fsx_status s = check_tick_args(h, k_cache, v_cache, d_offsets, B, d_frames, d_waypoints);
+  if (s != FSX_OK) return s;
+  std::lock_guard<std::mutex> lock(h->mu);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  s = prepare_tick(h, k_cache, v_cache, d_offsets, d_frames, d_waypoints, st);
+  if (s != FSX_OK) return s;
+  cudaGraphExec_t exec = nullptr;
+  s = get_graph(h, B, h->timing, &exec);
+  if (s != FSX_OK) return s;
+  FSX_CUDA(cudaGraphLaunch(exec, st));
+  h->timed_pending = h->timing;
+  return finish_tick(h, st);
+}
+
+fsx_status fsx_tick_host(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                         const int64_t* h_offsets, int B, const void* h_frames, float* h_waypoints, void* stream) {
+  fsx_status s = check_tick_args(h, k_cache, v_cache, h_offsets, B, h_frames, h_waypoints);
+  if (s != FSX_OK) return s;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  {
+    std::lock_guard<std::mutex> lock(h->mu);
+    FSX_CUDA(cudaSetDevice(h->device));
+    if (h->has_last && h->last_stream != st) FSX_CUDA(cudaStreamWaitEvent(st, h->last_tick, 0));
+    const size_t fbytes = static_cast<size_t>(B) * h->cfg.n_frame * h->cfg.d_model *
+                          (h->cfg.frame_dtype == FSX_BF16 ? 2 : 4);
+    FSX_CUDA(cudaMemcpyAsync(h->st_offsets, h_offsets, (B + 1) * sizeof(int64_t), cudaMemcpyHostToDevice, st));
+    if (fbytes) FSX_CUDA(cudaMemcpyAsync(h->st_frames, h_frames, fbytes, cudaMemcpyHostToDevice, st));
+  }
+  s = fsx_tick(h, k_cache, v_cache, h->st_offsets, B, h->st_frames, h->st_waypoints, stream);
+  if (s != FSX_OK) return s;
+  FSX_CUDA(cudaMemcpyAsync(h_waypoints, h->st_waypoints,
+                           static_cast<size_t>(B) * h->cfg.n_waypoints * 2 * sizeof(float), cudaMemcpyDeviceToHost, st));
+  FSX_CUDA(cudaStreamSynchronize(st));
+  return FSX_OK;
+}
+
+fsx_status fsx_tick_debug(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                          const int64_t* d_offsets, int B, const void* d_frames, float* d_waypoints,
+                          void* d_attn_out, void* stream) {
+  fsx_status s = check_tick_args(h, k_cache, v_cache, d_offsets, B, d_frames, d_waypoints);
+  if (s != FSX_OK) return s;
+  if (!d_attn_out) return fail(FSX_ERR_INVALID_ARG, "d_attn_out is NULL");
+  std::lock_guard<std::mutex> lock(h->mu);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  s = prepare_tick(h, k_cache, v_cache, d_offsets, d_frames, d_waypoints, st);
+  if (s != FSX_OK) return s;
+  s = enqueue_tick(h, B, st, static_cast<__half*>(d_attn_out), false);
+  if (s != FSX_OK) return s;
+  return finish_tick(h, st);
+}
+
+fsx_status fsx_get_status(fsx_handle h, void* stream) {
+  if (!h) return fail(FSX_ERR_INVALID_ARG, "handle is NULL");
+  std::lock_guard<std::mutex> lock(h->mu);
+  FSX_CUDA(cudaSetDevice(h->device));
+  FSX_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  int v = 0;
+  FSX_CUDA(cudaMemcpyAsync(&v, h->status, sizeof(int), cudaMemcpyDeviceToHost, h->cap_stream));
+  FSX_CUDA(cudaMemsetAsync(h->status, 0, sizeof(int), h->cap_stream));
+  FSX_CUDA(cudaStreamSynchronize(h->cap_stream));
+  if (v == 0) return FSX_OK;
+  if (v == FSX_ERR_TIMEOUT) return fail(FSX_ERR_TIMEOUT, "a device-side wait timed out");
+  return fail(FSX_ERR_DEVICE_ARG, "device-side argument check failed (cache offsets)");
+}
+
+void fsx_destroy(fsx_handle h) { free_handle(h); }
+
+long long fsx_weight_bytes(fsx_handle h) { return h ? h->weight_bytes : 0; }
+
+int fsx_tick_launches(fsx_handle h, int B) {
+  if (!h || B < 1) return 0;
+  return 2 + h->cfg.n_layers * (4 + fsx::attention_launch_count(attention_splits(h, B)));
+}
+
+fsx_status fsx_set_kernel_timing(fsx_handle h, int enable, int kclass) {
+  if (!h) return fail(FSX_ERR_INVALID_ARG, "handle is NULL");
+  if (kclass < kClassQkv || kclass > kClassDown) return fail(FSX_ERR_INVALID_ARG, "kernel class %d unknown", kclass);
+  std::lock_guard<std::mutex> lock(h->mu);
+  if (enable && kclass != h->timing_class) {
+    for (auto& kv : h->timed_graphs) cudaGraphExecDestroy(kv.second);
+    h->timed_graphs.clear();
+  }
+  h->timing = enable != 0;
+  h->timing_class = kclass;
+  return FSX_OK;
+}
+
+fsx_status fsx_kernel_time(fsx_handle h, float* ms, int* launches) {
+  if (!h || !ms || !launches) return fail(FSX_ERR_INVALID_ARG, "NULL argument");
+  std::lock_guard<std::mutex> lock(h->mu);
+  if (!h->timed_pending || h->timed_pairs == 0) return fail(FSX_ERR_INVALID_ARG, "no timed tick recorded");
+  FSX_CUDA(cudaSetDevice(h->device));
+  FSX_CUDA(cudaEventSynchronize(h->tev[2 * h->timed_pairs - 1]));
+  float total = 0.f;
+  for (int i = 0; i < h->timed_pairs; ++i) {
+    float t = 0.f;
+    FSX_CUDA(cudaEventElapsedTime(&t, h->tev[2 * i], h->tev[2 * i + 1]));
+    total += t;
+  }
+  *ms = total;
+  *launches = h->timed_pairs;
+  return FSX_OK;
+}
+
+size_t fsx_attention_workspace_bytes(int B, int n_heads, int n_q, int n_splits) {
+  (void)n_q;
+  if (B < 1 || n_heads < 1 || n_splits < 1) return 0;
+  return 256 + fsx::attention_workspace_bytes(B, n_heads, n_splits);
+}
+
+fsx_status fsx_attention(const void* d_q, long long q_stride, const void* d_k_own, const void* d_v_own,
+                         long long own_stride, int n_q, int n_own, const void* d_k_cache, const void* d_v_cache,
+                         int cache_dtype, const int64_t* d_offsets, int B, int n_heads, int head_dim, int n_splits,
+                         void* d_out, float* d_lse, void* d_workspace, size_t workspace_bytes, void* stream) {
+  g_err[0] = '\0';
+  if (!d_q || !d_offsets || !d_out || !d_k_cache || !d_v_cache) return fail(FSX_ERR_INVALID_ARG, "NULL pointer argument");
+  if (n_own > 0 && (!d_k_own || !d_v_own)) return fail(FSX_ERR_INVALID_ARG, "own key/value pointers are NULL");
+  if (head_dim != fsx::kHeadDim) return fail(FSX_ERR_UNSUPPORTED, "head_dim must be 128");
+  if (n_q < 1 || n_q > fsx::kTokTile) return fail(FSX_ERR_INVALID_ARG, "n_q must be in 1..48");
+  if (n_own < 0 || B < 1 || n_heads < 1) return fail(FSX_ERR_INVALID_ARG, "n_own >= 0, B >= 1, n_heads >= 1");
+  if (n_splits < 1 || n_splits > fsx::kMaxSplits) return fail(FSX_ERR_INVALID_ARG, "n_splits must be in 1..64");
+  if (cache_dtype != FSX_F32 && cache_dtype != FSX_BF16) return fail(FSX_ERR_INVALID_ARG, "bad cache_dtype");
+  if (q_stride < static_cast<long long>(n_heads) * head_dim || (n_own > 0 && own_stride < static_cast<long long>(n_heads) * head_dim) ||
+      (q_stride % 8) != 0 || (own_stride % 8) != 0)
+    return fail(FSX_ERR_INVALID_ARG, "strides must cover n_heads*head_dim and be multiples of 8");
+  const size_t need = fsx_attention_workspace_bytes(B, n_heads, n_q, n_splits);
+  if (!d_workspace || workspace_bytes < need)
+    return fail(FSX_ERR_INVALID_ARG, "workspace of %zu bytes required", need);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int* status = static_cast<int*>(d_workspace);  // first 256 bytes: status word
+  float* part = reinterpret_cast<float*>(static_cast<unsigned char*>(d_workspace) + 256);
+  FSX_CUDA(cudaMemsetAsync(status, 0, sizeof(int), st));
+  FSX_CUDA(fsx::attention_set_attributes());
+  fsx::AttnArgs a{};
+  a.q = static_cast<const __half*>(d_q);
+  a.q_stride = q_stride;
+  a.k_own = static_cast<const __half*>(d_k_own);
+  a.v_own = static_cast<const __half*>(d_v_own);
+  a.own_stride = own_stride;
+  a.n_q = n_q;
+  a.n_own = n_own;
+  a.k_cache = d_k_cache;
+  a.v_cache = d_v_cache;
+  a.targs = nullptr;
+  a.layer = 0;
+  a.offsets = d_offsets;
+  a.max_total = (1ll << 62);
+  a.n_heads = n_heads;
+  a.n_splits = n_splits;
+  a.out = static_cast<__half*>(d_out);
+  a.out_stride = static_cast<long long>(n_heads) * head_dim;
+  a.lse = d_lse;
+  a.part_o = part;
+  a.part_lse = part + static_cast<size_t>(B) * n_heads * n_splits * fsx::kTokTile * fsx::kHeadDim;
+  a.status = status;
+  FSX_CUDA(fsx::launch_attention(a, B, cache_dtype, st, false));
+  return FSX_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,291 @@
+// Weight-streaming projection GEMMs of the expert layer (Sec. 3.1: the
+// rectangular W_q/W_k/W_v projections, the output projection W_o and the
+// SwiGLU block), for the small token counts of a tick (M = 42 B rows).
+//
+// Y[M, N] = A[M, K] . W[N, K]^T on fp16 tensor cores (mma.sync m16n8k16, fp32
+// accumulation) with the weights as the 16-row operand ("swap-AB"), so a
+// 48-token tile is six n8 column tiles and every weight byte is used for six
+// MMAs. Each CTA owns nb x 16 weight rows and a K range; its weight tile is a
+// contiguous run of fragment-ordered blocks that one thread fetches with bulk
+// copies (mbarrier completion) BEFORE waiting on the previous kernel, so the
+// weight stream overlaps the tail of the preceding step. The activation tile
+// (48 x K range, fp16) is staged in shared memory by the prologue, either as
+// RMSNorm(x) * gamma from the fp32 residual stream or as a copy of fp16 rows.
+// Warps split the K range; a shared-memory reduction combines them and the
+// epilogue stores fp16, adds fp32 partials into the residual stream (split-K),
+// or applies the SwiGLU gate to row pairs packed next to each other.
+#include "device_util.cuh"
+#include "kernels.h"
+
+namespace fsx {
+
+namespace {
+
+constexpr int kThreads = 128;   // 4 warps
+constexpr int kRedStride = kTokTile + 4;
+
+__host__ __device__ constexpr int a_stride(int ks) { return ks + 8; }  // halves, 16-byte row pad
+
+__host__ __device__ inline size_t gemm_smem_bytes(int nb, int ks) {
+  return 128 + static_cast<size_t>(nb) * (ks / 16) * 512 + static_cast<size_t>(kTokTile) * a_stride(ks) * 2 +
+         static_cast<size_t>(4) * (16 * nb) * kRedStride * 4;
+}
+
+template <int NB, int PRO, int EPI>
+__global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
+  constexpr int NT = 16 * NB;
+  extern __shared__ __align__(128) unsigned char smem[];
+  const int ks = p.ks;
+  const int lda_s = a_stride(ks);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem);
+  uint4* sW = reinterpret_cast<uint4*>(smem + 128);
+  __half* sA = reinterpret_cast<__half*>(smem + 128 + static_cast<size_t>(NB) * (ks / 16) * 512);
+  float* sR = reinterpret_cast<float*>(sA + static_cast<size_t>(kTokTile) * lda_s);
+
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
+  const int nb0 = blockIdx.x * NB;
+  const int k0 = blockIdx.y * ks;
+  const int kl = min(ks, p.K - k0);
+  const int kb_total = p.K / 16;
+
+  pdl_launch_dependents();
+  if (tid == 0) {
+    mbar_init(bar, 1);
+    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(NB * (kl / 16) * 512));
+#pragma unroll
+    for (int j = 0; j < NB; ++j) {
+      const uint4* src = p.w + (static_cast<size_t>(nb0 + j) * kb_total + k0 / 16) * 32;
+      bulk_g2s(sW + static_cast<size_t>(j) * (ks / 16) * 32, src, static_cast<uint32_t>((kl / 16) * 512), bar);
+    }
+  }
+  __syncthreads();  // barrier initialised before anyone polls it
+  pdl_wait();
+  const bool weights_ok = mbar_wait(bar, 0, p.status);
+  if (!weights_ok || *reinterpret_cast<volatile int*>(p.status) != 0) return;
+
+  const int n_mtiles = (p.M + kTokTile - 1) / kTokTile;
+  const int mt_begin = blockIdx.z * p.m_tiles_per_cta;
+  const int mt_end = min(n_mtiles, mt_begin + p.m_tiles_per_cta);
+
+  for (int mt = mt_begin; mt < mt_end; ++mt) {
+    const int m0 = mt * kTokTile;
+    // ---------------- prologue: activation tile -> sA (fp16)
+    if (PRO == kProNorm) {
+      for (int r = warp; r < kTokTile; r += 4) {
+        const int m = m0 + r;
+        __half* dst = sA + static_cast<size_t>(r) * lda_s;
+        if (m < p.M) {
+          const float* xr = p.x + static_cast<size_t>(m) * p.ldx;
+          float ss = 0.f;
+          for (int c = lane * 4; c < p.K; c += 128) {
+            const float4 v = *reinterpret_cast<const float4*>(xr + c);
+            ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+          }
+          ss = warp_sum(ss);
+          const float rstd = rsqrtf(ss / static_cast<float>(p.K) + 1e-6f);
+          for (int c = lane * 4; c < kl; c += 128) {
+            const float4 v = *reinterpret_cast<const float4*>(xr + k0 + c);
+            const float4 g = *reinterpret_cast<const float4*>(p.gamma + k0 + c);
+            uint2 packed;
+            packed.x = pack_half2(v.x * rstd * g.x, v.y * rstd * g.y);
+            packed.y = pack_half2(v.z * rstd * g.z, v.w * rstd * g.w);
+            *reinterpret_cast<uint2*>(dst + c) = packed;
+          }
+        } else {
+          for (int c = lane * 4; c < kl; c += 128) *reinterpret_cast<uint2*>(dst + c) = make_uint2(0u, 0u);
+        }
+      }
+    } else {
+      const int cpr = kl / 8;  // 16-byte chunks per row
+      for (int i = tid; i < kTokTile * cpr; i += kThreads) {
+        const int r = i / cpr;
+        const int c = (i - r * cpr) * 8;
+        const int m = m0 + r;
+        __half* dst = sA + static_cast<size_t>(r) * lda_s + c;
+        if (m < p.M) {
+          cp_async_16(smem_addr(dst), p.a + static_cast<size_t>(m) * p.lda + k0 + c);
+        } else {
+          *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+      cp_async_commit();
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+
+    // ---------------- tensor-core main loop: warp w takes 64-wide K groups w, w+4, ...
+    float acc[NB][6][4];
+#pragma unroll
+    for (int j = 0; j < NB; ++j)
+#pragma unroll
+      for (int t = 0; t < 6; ++t)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc[j][t][e] = 0.f;
+
+    const int n_groups = kl / 64;
+    for (int g = warp; g < n_groups; g += 4) {
+      uint32_t bfr[6][4][2];
+#pragma unroll
+      for (int t = 0; t < 6; ++t) {
+#pragma unroll
+        for (int kp = 0; kp < 2; ++kp) {
+          const __half* src = sA + static_cast<size_t>(t * 8 + (lane & 7)) * lda_s + g * 64 + kp * 32 + (lane >> 3) * 8;
+          ldsm_x4(bfr[t][2 * kp][0], bfr[t][2 * kp][1], bfr[t][2 * kp + 1][0], bfr[t][2 * kp + 1][1], smem_addr(src));
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < NB; ++j) {
+#pragma unroll
+        for (int kb = 0; kb < 4; ++kb) {
+          const uint4 af = sW[(static_cast<size_t>(j) * (ks / 16) + g * 4 + kb) * 32 + lane];
+#pragma unroll
+          for (int t = 0; t < 6; ++t) mma_f16_16816(acc[j][t], af.x, af.y, af.z, af.w, bfr[t][kb][0], bfr[t][kb][1]);
+        }
+      }
+    }
+
+    // ---------------- cross-warp reduction through shared memory
+#pragma unroll
+    for (int j = 0; j < NB; ++j) {
+#pragma unroll
+      for (int t = 0; t < 6; ++t) {
+        const int n = j * 16 + (lane >> 2);
+        const int m = t * 8 + 2 * (lane & 3);
+        float* r0 = sR + (static_cast<size_t>(warp) * NT + n) * kRedStride + m;
+        float* r1 = r0 + 8 * kRedStride;
+        *reinterpret_cast<float2*>(r0) = make_float2(acc[j][t][0], acc[j][t][1]);
+        *reinterpret_cast<float2*>(r1) = make_float2(acc[j][t][2], acc[j][t][3]);
+      }
+    }
+    __syncthreads();
+
+    auto red = [&](int n, int m) -> float {
+      const float* r = sR + static_cast<size_t>(n) * kRedStride + m;
+      return r[0] + r[NT * kRedStride] + r[2 * NT * kRedStride] + r[3 * NT * kRedStride];
+    };
+
+    // ---------------- epilogue
+    if (EPI == kEpiStore) {
+      constexpr int NP = NT / 2;
+      for (int i = tid; i < NP * kTokTile; i += kThreads) {
+        const int n = (i % NP) * 2;
+        const int m = i / NP;
+        if (m0 + m < p.M) {
+          const uint32_t v = pack_half2(red(n, m), red(n + 1, m));
+          *reinterpret_cast<uint32_t*>(p.y + static_cast<size_t>(m0 + m) * p.ldy + nb0 * 16 + n) = v;
+        }
+      }
+    } else if (EPI == kEpiAtomic) {
+      constexpr int NQ = NT / 4;
+      for (int i = tid; i < NQ * kTokTile; i += kThreads) {
+        const int n = (i % NQ) * 4;
+        const int m = i / NQ;
+        if (m0 + m < p.M) {
+          const float4 v = make_float4(red(n, m), red(n + 1, m), red(n + 2, m), red(n + 3, m));
+          atomicAdd(reinterpret_cast<float4*>(p.xo + static_cast<size_t>(m0 + m) * p.ldxo + nb0 * 16 + n), v);
+        }
+      }
+    } else {  // kEpiSwiglu: block j rows 0..7 = gate of h columns (nb0+j)*8 + r, rows 8..15 = up
+      constexpr int NH = NB * 8;
+      for (int i = tid; i < NH * kTokTile; i += kThreads) {
+        const int hc = i % NH;
+        const int m = i / NH;
+        if (m0 + m < p.M) {
+          const int j = hc >> 3;
+          const int r = hc & 7;
+          const float g = red(j * 16 + r, m);
+          const float u = red(j * 16 + 8 + r, m);
+          const float hval = g / (1.f + __expf(-g)) * u;
+          p.y[static_cast<size_t>(m0 + m) * p.ldy + nb0 * 8 + hc] = __float2half_rn(hval);
+        }
+      }
+    }
+    __syncthreads();  // sA / sR reused by the next m-tile
+  }
+}
+
+template <int NB, int PRO, int EPI>
+const void* kernel_ptr() {
+  return reinterpret_cast<const void*>(&gemm_ws_kernel<NB, PRO, EPI>);
+}
+
+const void* select_kernel(int nb, int pro, int epi) {
+#define FSX_SEL(NB_, PRO_, EPI_) \
+  if (nb == NB_ && pro == PRO_ && epi == EPI_) return kernel_ptr<NB_, PRO_, EPI_>();
+  FSX_SEL(1, kProNorm, kEpiStore)
+  FSX_SEL(2, kProNorm, kEpiStore)
+  FSX_SEL(1, kProNorm, kEpiSwiglu)
+  FSX_SEL(2, kProNorm, kEpiSwiglu)
+  FSX_SEL(1, kProCopy, kEpiAtomic)
+  FSX_SEL(2, kProCopy, kEpiAtomic)
+  FSX_SEL(1, kProCopy, kEpiStore)
+  FSX_SEL(2, kProCopy, kEpiStore)
+#undef FSX_SEL
+  return nullptr;
+}
+
+}  // namespace
+
+cudaError_t gemm_set_attributes() {
+  const int nbs[2] = {1, 2};
+  const int pros[2] = {kProNorm, kProCopy};
+  const int epis[3] = {kEpiStore, kEpiAtomic, kEpiSwiglu};
+  for (int nb : nbs)
+    for (int pro : pros)
+      for (int epi : epis) {
+        const void* fn = select_kernel(nb, pro, epi);
+        if (!fn) continue;
+        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, 220 * 1024);
+        if (e != cudaSuccess) return e;
+      }
+  return cudaSuccess;
+}
+
+GemmPlan plan_gemm(int n_rows, int K, int M, int nb, int ks, int prologue, int epilogue, int sm_count) {
+  GemmPlan pl{};
+  pl.nb = nb;
+  pl.ks = ks;
+  pl.prologue = prologue;
+  pl.epilogue = epilogue;
+  const int nx = n_rows / (16 * nb);
+  const int ny = (K + ks - 1) / ks;
+  const int m_tiles = (M + kTokTile - 1) / kTokTile;
+  int nz = (4 * sm_count) / (nx * ny);
+  if (nz < 1) nz = 1;
+  if (nz > m_tiles) nz = m_tiles;
+  const int per = (m_tiles + nz - 1) / nz;
+  nz = (m_tiles + per - 1) / per;
+  pl.grid = dim3(nx, ny, nz);
+  pl.smem = gemm_smem_bytes(nb, ks);
+  return pl;
+}
+
+cudaError_t launch_gemm(const GemmPlan& pl, const GemmArgs& args_in, cudaStream_t stream, bool pdl) {
+  GemmArgs args = args_in;
+  args.ks = pl.ks;
+  const int m_tiles = (args.M + kTokTile - 1) / kTokTile;
+  args.m_tiles_per_cta = (m_tiles + static_cast<int>(pl.grid.z) - 1) / static_cast<int>(pl.grid.z);
+  const void* fn = select_kernel(pl.nb, pl.prologue, pl.epilogue);
+  if (!fn) return cudaErrorInvalidValue;
+  void* kargs[] = {&args};
+  return launch_ex(fn, pl.grid, dim3(kThreads), pl.smem, stream, pdl, kargs);
+}
+
+cudaError_t launch_ex(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool pdl,
+                      void** args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelExC(&cfg, fn, args);
+}
+
+}  // namespace fsx

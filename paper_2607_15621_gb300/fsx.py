@@ -1,0 +1,224 @@
+"""Thin ctypes binding of libfsx.so (include/fsx.h): argument marshalling only.
+
+Every step of the tick runs in the library's CUDA kernels; this module only
+turns torch tensors / numpy arrays into pointers, sizes and a cudaStream_t.
+Importing it fails loudly when the compiled library is missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Sequence
+
+import numpy as np
+
+from .synth import Dims
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "_lib", "libfsx.so")
+
+FSX_OK = 0
+FSX_ERR_INVALID_ARG = 1
+FSX_ERR_UNSUPPORTED = 2
+FSX_ERR_OOM = 3
+FSX_ERR_CUDA = 4
+FSX_ERR_TIMEOUT = 5
+FSX_ERR_DEVICE_ARG = 6
+FSX_F32 = 0
+FSX_BF16 = 1
+
+KCLASS = {"qkv": 0, "attention": 1, "out_proj": 2, "gate_up": 3, "down": 4}
+
+
+class FsxError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"fsx status {status}: {message}")
+        self.status = status
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int), ("d_model", ctypes.c_int), ("n_heads", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("d_ff", ctypes.c_int), ("n_action", ctypes.c_int),
+                ("n_frame", ctypes.c_int), ("n_waypoints", ctypes.c_int), ("max_batch", ctypes.c_int),
+                ("max_total_cache_tokens", ctypes.c_longlong), ("cache_dtype", ctypes.c_int),
+                ("frame_dtype", ctypes.c_int)]
+
+
+_WEIGHT_FIELDS = ["act_emb", "pos_emb", "attn_norm", "wq", "wk", "wv", "wo", "mlp_norm", "w_gate",
+                  "w_up", "w_down", "final_norm", "head_w", "head_b"]
+
+
+class Weights(ctypes.Structure):
+    _fields_ = [(name, ctypes.POINTER(ctypes.c_float)) for name in _WEIGHT_FIELDS]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with paper_2607_15621_gb300.build.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i32, i64p = ctypes.c_void_p, ctypes.c_int, ctypes.POINTER(ctypes.c_int64)
+    vpp = ctypes.POINTER(ctypes.c_void_p)
+    fp = ctypes.POINTER(ctypes.c_float)
+    sig = {
+        "fsx_create": (i32, [ctypes.POINTER(Config), ctypes.POINTER(Weights), i32, ctypes.POINTER(vp)]),
+        "fsx_tick": (i32, [vp, vpp, vpp, vp, i32, vp, vp, vp]),
+        "fsx_tick_host": (i32, [vp, vpp, vpp, vp, i32, vp, vp, vp]),
+        "fsx_tick_debug": (i32, [vp, vpp, vpp, vp, i32, vp, vp, vp, vp]),
+        "fsx_get_status": (i32, [vp, vp]),
+        "fsx_last_error": (ctypes.c_char_p, []),
+        "fsx_destroy": (None, [vp]),
+        "fsx_weight_bytes": (ctypes.c_longlong, [vp]),
+        "fsx_tick_launches": (i32, [vp, i32]),
+        "fsx_set_kernel_timing": (i32, [vp, i32, i32]),
+        "fsx_kernel_time": (i32, [vp, fp, ctypes.POINTER(ctypes.c_int)]),
+        "fsx_attention_workspace_bytes": (ctypes.c_size_t, [i32, i32, i32, i32]),
+        "fsx_attention": (i32, [vp, ctypes.c_longlong, vp, vp, ctypes.c_longlong, i32, i32, vp, vp, i32,
+                                vp, i32, i32, i32, i32, vp, vp, vp, ctypes.c_size_t, vp]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _lib = _load()
+    return _lib
+
+
+def declared_symbols() -> list[str]:
+    return ["fsx_create", "fsx_tick", "fsx_tick_host", "fsx_tick_debug", "fsx_get_status", "fsx_last_error",
+            "fsx_destroy", "fsx_weight_bytes", "fsx_tick_launches", "fsx_set_kernel_timing",
+            "fsx_kernel_time", "fsx_attention_workspace_bytes", "fsx_attention"]
+
+
+def last_error() -> str:
+    return lib().fsx_last_error().decode()
+
+
+def check(status: int):
+    if status != FSX_OK:
+        raise FsxError(status, last_error())
+
+
+def _ptr(t) -> int:
+    """Device or host address of a torch tensor / numpy array (None -> 0)."""
+    if t is None:
+        return 0
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _ptr_array(tensors: Sequence) -> ctypes.Array:
+    arr = (ctypes.c_void_p * len(tensors))()
+    for i, t in enumerate(tensors):
+        arr[i] = _ptr(t)
+    return arr
+
+
+def make_config(dims: Dims, max_batch: int, max_total_cache_tokens: int, cache_dtype: str = "bf16",
+                frame_dtype: str = "bf16") -> Config:
+    code = {"fp32": FSX_F32, "bf16": FSX_BF16}
+    return Config(dims.n_layers, dims.d_model, dims.n_heads, dims.head_dim, dims.d_ff, dims.n_action,
+                  dims.n_frame, dims.n_waypoints, max_batch, max_total_cache_tokens,
+                  code[cache_dtype], code[frame_dtype])
+
+
+def make_weights(weights: dict):
+    """ctypes struct of host fp32 pointers plus the contiguous arrays it points to."""
+    keep = {k: np.ascontiguousarray(weights[k], dtype=np.float32) for k in _WEIGHT_FIELDS}
+    st = Weights(*[keep[k].ctypes.data_as(ctypes.POINTER(ctypes.c_float)) for k in _WEIGHT_FIELDS])
+    return st, keep
+
+
+class Expert:
+    """Owns one fsx handle (weights uploaded at construction)."""
+
+    def __init__(self, dims: Dims, weights: dict, max_batch: int, max_total_cache_tokens: int,
+                 cache_dtype: str = "bf16", frame_dtype: str = "bf16", device: int = 0):
+        self.dims = dims
+        self.cfg = make_config(dims, max_batch, max_total_cache_tokens, cache_dtype, frame_dtype)
+        wst, keep = make_weights(weights)
+        h = ctypes.c_void_p()
+        check(lib().fsx_create(ctypes.byref(self.cfg), ctypes.byref(wst), device, ctypes.byref(h)))
+        self.h = h
+        del keep
+
+    def close(self):
+        if getattr(self, "h", None) and self.h.value:
+            lib().fsx_destroy(self.h)
+            self.h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def tick(self, k_layers, v_layers, offsets, frames, out, stream=None):
+        B = int(frames.shape[0])
+        check(lib().fsx_tick(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(offsets), B,
+                             _ptr(frames), _ptr(out), _stream(stream)))
+        return out
+
+    def tick_host(self, k_layers, v_layers, offsets_host: np.ndarray, frames_host, out_host: np.ndarray,
+                  stream=None):
+        B = int(frames_host.shape[0])
+        check(lib().fsx_tick_host(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(offsets_host), B,
+                                  _ptr(frames_host), _ptr(out_host), _stream(stream)))
+        return out_host
+
+    def tick_debug(self, k_layers, v_layers, offsets, frames, out, attn_out, stream=None):
+        B = int(frames.shape[0])
+        check(lib().fsx_tick_debug(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(offsets), B,
+                                   _ptr(frames), _ptr(out), _ptr(attn_out), _stream(stream)))
+        return out, attn_out
+
+    def status(self, stream=None) -> int:
+        return lib().fsx_get_status(self.h, _stream(stream))
+
+    def weight_bytes(self) -> int:
+        return int(lib().fsx_weight_bytes(self.h))
+
+    def launches(self, B: int) -> int:
+        return int(lib().fsx_tick_launches(self.h, B))
+
+    def set_kernel_timing(self, enable: bool, kclass: str = "qkv"):
+        check(lib().fsx_set_kernel_timing(self.h, int(enable), KCLASS[kclass]))
+
+    def kernel_time(self):
+        ms = ctypes.c_float()
+        n = ctypes.c_int()
+        check(lib().fsx_kernel_time(self.h, ctypes.byref(ms), ctypes.byref(n)))
+        return float(ms.value), int(n.value)
+
+
+def attention_workspace_bytes(B: int, n_heads: int, n_q: int, n_splits: int) -> int:
+    return int(lib().fsx_attention_workspace_bytes(B, n_heads, n_q, n_splits))
+
+
+def attention(q, q_stride, k_own, v_own, own_stride, n_q, n_own, k_cache, v_cache, cache_dtype, offsets, B,
+              n_heads, n_splits, out, lse, workspace, stream=None):
+    """Eq. 1 alone through the C ABI (fp16 tensors, int64 offsets, caller scratch)."""
+    code = {"fp32": FSX_F32, "bf16": FSX_BF16}[cache_dtype]
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    check(lib().fsx_attention(_ptr(q), q_stride, _ptr(k_own), _ptr(v_own), own_stride, n_q, n_own,
+                              _ptr(k_cache), _ptr(v_cache), code, _ptr(offsets), B, n_heads, 128, n_splits,
+                              _ptr(out), _ptr(lse), _ptr(workspace), ws_bytes, _stream(stream)))
+    return out

@@ -1,0 +1,147 @@
+"""Whole expert tick through the C ABI against the fp64 oracle on the same
+seeded inputs: per-layer Eq. 1 outputs (2e-2 * max|ref| per row) and waypoints
+(1e-2 relative L2), at every workload shape, plus the tick's invariants and
+error paths."""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_15621_gb300 import fsx, synth
+
+import fsx_cases as fc
+
+pytestmark = pytest.mark.gpu
+
+SMALL = synth.Dims(n_layers=4)
+
+
+def _parity(case, vehicles=None, max_batch=None):
+    ex = case.expert(max_batch)
+    try:
+        wp, att = fc.run_debug_tick(ex, case)
+        wp_graph = fc.run_tick(ex, case)
+    finally:
+        ex.close()
+    assert np.isfinite(wp).all()
+    # graph replay and the kernel-by-kernel debug path compute the same tick
+    assert np.linalg.norm(wp_graph - wp) <= 1e-3 * np.linalg.norm(wp)
+    worst = []
+    for b in (range(case.B) if vehicles is None else vehicles):
+        worst.append(fc.check_vehicle(case, b, wp, att))
+    return worst
+
+
+def test_tick_small_ragged_with_empty_cache():
+    """4 layers of the full-width expert, 3 vehicles, L_b = 0 / 70 / 150."""
+    _parity(fc.Case(SMALL, [0, 70, 150], "bf16", seed=1))
+
+
+def test_tick_fp32_inputs_b1_l96():
+    """fp32 weights, cache and frames; B=1, L=96 (32 instruction + 16 frames x 4)."""
+    _parity(fc.Case(synth.EXPERT, synth.cache_lengths("fp32_b1_l96"), "fp32"))
+
+
+def test_tick_bf16_b1_l224():
+    """bf16 inputs, B=1, L=224 (64 instruction + 40 frames x 4): the paper-shaped latency case."""
+    _parity(fc.Case(synth.EXPERT, synth.cache_lengths("bf16_b1_l224"), "bf16"))
+
+
+@pytest.mark.parametrize("length", [512, 4096])
+def test_tick_bf16_history_sweep(length):
+    _parity(fc.Case(synth.EXPERT, [length], "bf16"))
+
+
+def test_tick_bf16_b16_ragged():
+    """B=16 vehicles with L_b ~ U[96, 480] sharing the expert weights."""
+    _parity(fc.Case(synth.EXPERT, synth.cache_lengths("bf16_b16_ragged"), "bf16"))
+
+
+def test_tick_bf16_b128_ragged_sampled():
+    """B=128, L_b ~ U[64, 2048] (~71 GB of cache): the whole batch runs on the
+    GPU; the oracle checks 6 sampled vehicles incl. the shortest and longest."""
+    lengths = synth.cache_lengths("bf16_b128_ragged")
+    case = fc.Case(synth.EXPERT, lengths, "bf16", gen_device="cuda")
+    rng = np.random.default_rng(0)
+    pick = sorted({int(np.argmin(lengths)), int(np.argmax(lengths)), *rng.choice(len(lengths), 4, replace=False)})
+    _parity(case, vehicles=pick)
+
+
+def test_cache_is_never_written_and_vehicles_are_independent():
+    case = fc.Case(SMALL, [40, 90, 17], "bf16", seed=2)
+    before = [(k.clone(), v.clone()) for k, v in zip(case.k, case.v)]
+    ex = case.expert()
+    try:
+        wp = fc.run_tick(ex, case)
+        for (k0, v0), k1, v1 in zip(before, case.k, case.v):
+            assert torch.equal(k0.view(torch.int16), k1.view(torch.int16))
+            assert torch.equal(v0.view(torch.int16), v1.view(torch.int16))
+        lo, hi = int(case.offsets_np[1]), int(case.offsets_np[2])
+        for k in case.k:
+            k[lo:hi] = -k[lo:hi]
+        wp2 = fc.run_tick(ex, case)
+    finally:
+        ex.close()
+    assert np.max(np.abs(wp2[[0, 2]] - wp[[0, 2]])) <= 1e-4 * np.max(np.abs(wp[[0, 2]]))
+    assert np.max(np.abs(wp2[1] - wp[1])) > 1e-3
+
+
+def test_tick_host_buffers_match_device_tick():
+    case = fc.Case(SMALL, [33, 0], "bf16", seed=3)
+    ex = case.expert(max_batch=4)
+    try:
+        wp = fc.run_tick(ex, case)
+        out = np.zeros((case.B, case.dims.n_waypoints, 2), dtype=np.float32)
+        ex.tick_host(case.k, case.v, case.offsets_np.copy(), case.frames.cpu().contiguous(), out)
+    finally:
+        ex.close()
+    assert np.linalg.norm(out - wp) <= 1e-3 * np.linalg.norm(wp)
+
+
+def test_batch_sizes_reuse_one_handle():
+    """One handle serves several B (one captured graph per B)."""
+    case = fc.Case(SMALL, [20, 60, 5, 0, 33], "bf16", seed=4)
+    ex = case.expert(max_batch=8)
+    try:
+        full = fc.run_tick(ex, case)
+        sub = fc.Case(SMALL, [20, 60], "bf16", seed=4)
+        part = fc.run_tick(ex, sub)
+    finally:
+        ex.close()
+    ref0, _ = case.oracle_vehicle(0, capture=True)
+    assert np.linalg.norm(full[0] - ref0[0]) <= fc.WAYPOINT_TOL * np.linalg.norm(ref0[0])
+    assert np.isfinite(part).all()
+
+
+def test_device_side_offset_check_and_recovery():
+    case = fc.Case(SMALL, [30, 30], "bf16", seed=5)
+    ex = case.expert()
+    try:
+        bad = torch.tensor([0, 40, 20], device="cuda", dtype=torch.int64)
+        out = torch.full((2, case.dims.n_waypoints, 2), 123.0, device="cuda")
+        ex.tick(case.k, case.v, bad, case.frames, out)
+        assert ex.status() == fsx.FSX_ERR_DEVICE_ARG
+        assert torch.all(out == 123.0)  # the head never ran
+        beyond = torch.tensor([0, 30, 61], device="cuda", dtype=torch.int64)  # > max_total_cache_tokens
+        ex.tick(case.k, case.v, beyond, case.frames, out)
+        assert ex.status() == fsx.FSX_ERR_DEVICE_ARG
+        wp = fc.run_tick(ex, case)  # status was cleared by the read
+        assert np.isfinite(wp).all()
+    finally:
+        ex.close()
+
+
+def test_host_argument_errors_with_a_handle():
+    case = fc.Case(SMALL, [8], "bf16", seed=6)
+    ex = case.expert(max_batch=1)
+    try:
+        out = torch.empty(2, case.dims.n_waypoints, 2, device="cuda")
+        frames2 = torch.cat([case.frames, case.frames])
+        with pytest.raises(fsx.FsxError) as e:
+            ex.tick(case.k, case.v, case.offsets, frames2, out)
+        assert e.value.status == fsx.FSX_ERR_INVALID_ARG
+        with pytest.raises(fsx.FsxError):
+            ex.tick(case.k[:-1] + [None], case.v, case.offsets, case.frames, out)
+    finally:
+        ex.close()
