@@ -97,7 +97,8 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
  *   k_cache, v_cache : HOST arrays of n_layers DEVICE pointers; layer l points
  *                      to [total_tokens, n_heads, head_dim] rows of
  *                      cfg.cache_dtype, token-major, vehicle b owning rows
- *                      offsets[b] .. offsets[b+1]-1. Read only.
+ *                      offsets[b] .. offsets[b+1]-1. Read only. A layer
+ *                      pointer may be NULL only when every L_b is 0.
  *   d_offsets        : DEVICE int64 [B+1], non-decreasing, offsets[0] >= 0,
  *                      offsets[B] <= max_total_cache_tokens. L_b may be 0.
  *   B                : 1 .. max_batch.
@@ -105,8 +106,8 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
  *   d_waypoints      : DEVICE fp32 [B, n_waypoints, 2] output.
  * Enqueued on `stream` as one CUDA-graph launch (plus a small argument upload
  * when any pointer changed since the previous tick); no host synchronisation.
- * Device-side checks (offsets) set a sticky status read by fsx_get_status and
- * turn the remaining kernels of the tick into no-ops. A handle must not run
+ * Device-side checks (offsets) set a sticky status read by fsx_get_status;
+ * the rest of that tick then reads no cache row and writes no waypoint. A handle must not run
  * two ticks concurrently; ticks on different streams are serialised by the
  * handle. Must not be called while `stream` is being captured. */
 fsx_status fsx_tick(fsx_handle h, const void* const* k_cache, const void* const* v_cache,

@@ -101,7 +101,8 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
   }
   const long long o_lo = offs[b];
   const long long o_hi = offs[b + 1];
-  if (o_lo < 0 || o_hi < o_lo || o_hi > p.max_total) {  // never read outside the caller's cache
+  if (o_lo < 0 || o_hi < o_lo || o_hi > p.max_total ||
+      (o_hi > o_lo && (kc == nullptr || vc == nullptr))) {  // never read outside the caller's cache
     set_status(p.status, kStatusDeviceArg);
     return;
   }

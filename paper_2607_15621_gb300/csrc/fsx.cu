@@ -178,9 +178,9 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
   FSX_CUDA(fsx::launch_embed(ea, st, pdl));
 
   const fsx::GemmPlan pq = fsx::plan_gemm(3 * HD, d, M, 2, d, fsx::kProNorm, fsx::kEpiStore, h->sm_count);
-  const fsx::GemmPlan po = fsx::plan_gemm(d, HD, M, 2, 512, fsx::kProCopy, fsx::kEpiAtomic, h->sm_count);
+  const fsx::GemmPlan po = fsx::plan_gemm(d, HD, M, 2, 512, fsx::kProCopy, fsx::kEpiResidual, h->sm_count);
   const fsx::GemmPlan pg = fsx::plan_gemm(2 * F, d, M, 1, d, fsx::kProNorm, fsx::kEpiSwiglu, h->sm_count);
-  const fsx::GemmPlan pd = fsx::plan_gemm(d, F, M, 1, 256, fsx::kProCopy, fsx::kEpiAtomic, h->sm_count);
+  const fsx::GemmPlan pd = fsx::plan_gemm(d, F, M, 1, 256, fsx::kProCopy, fsx::kEpiResidual, h->sm_count);
   const int S = attention_splits(h, B);
 
   for (int l = 0; l < c.n_layers; ++l) {
@@ -322,8 +322,6 @@ fsx_status check_tick_args(fsx_handle_s* h, const void* const* k_cache, const vo
   if (!h) return fail(FSX_ERR_INVALID_ARG, "handle is NULL");
   if (B < 1 || B > h->cfg.max_batch) return fail(FSX_ERR_INVALID_ARG, "B=%d outside 1..max_batch=%d", B, h->cfg.max_batch);
   if (!k_cache || !v_cache) return fail(FSX_ERR_INVALID_ARG, "k_cache / v_cache pointer arrays are NULL");
-  for (int l = 0; l < h->cfg.n_layers; ++l)
-    if (!k_cache[l] || !v_cache[l]) return fail(FSX_ERR_INVALID_ARG, "cache pointer of layer %d is NULL", l);
   if (!offsets) return fail(FSX_ERR_INVALID_ARG, "offsets is NULL");
   if (!frames) return fail(FSX_ERR_INVALID_ARG, "frames is NULL");
   if (!waypoints) return fail(FSX_ERR_INVALID_ARG, "waypoints is NULL");
@@ -648,7 +646,7 @@ fsx_status fsx_attention(const void* d_q, long long q_stride, const void* d_k_ow
                          int cache_dtype, const int64_t* d_offsets, int B, int n_heads, int head_dim, int n_splits,
                          void* d_out, float* d_lse, void* d_workspace, size_t workspace_bytes, void* stream) {
   g_err[0] = '\0';
-  if (!d_q || !d_offsets || !d_out || !d_k_cache || !d_v_cache) return fail(FSX_ERR_INVALID_ARG, "NULL pointer argument");
+  if (!d_q || !d_offsets || !d_out) return fail(FSX_ERR_INVALID_ARG, "NULL pointer argument");
   if (n_own > 0 && (!d_k_own || !d_v_own)) return fail(FSX_ERR_INVALID_ARG, "own key/value pointers are NULL");
   if (head_dim != fsx::kHeadDim) return fail(FSX_ERR_UNSUPPORTED, "head_dim must be 128");
   if (n_q < 1 || n_q > fsx::kTokTile) return fail(FSX_ERR_INVALID_ARG, "n_q must be in 1..48");

@@ -12,10 +12,18 @@
 // (48 x K range, fp16) is staged in shared memory by the prologue, either as
 // RMSNorm(x) * gamma from the fp32 residual stream or as a copy of fp16 rows.
 // Warps split the K range; a shared-memory reduction combines them and the
-// epilogue stores fp16, adds fp32 partials into the residual stream (split-K),
-// or applies the SwiGLU gate to row pairs packed next to each other.
+// epilogue stores fp16, applies the SwiGLU gate to row pairs packed next to
+// each other, or adds the split-K sum into the fp32 residual stream. The K
+// splits of one output tile form a thread-block cluster: every CTA reduces
+// its warps into shared memory, and after a cluster barrier each CTA sums a
+// slice of the tile over all splits through distributed shared memory in
+// split order, so the residual update is deterministic and needs no atomics.
+#include <cooperative_groups.h>
+
 #include "device_util.cuh"
 #include "kernels.h"
+
+namespace cg = cooperative_groups;
 
 namespace fsx {
 
@@ -63,7 +71,10 @@ __global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
   __syncthreads();  // barrier initialised before anyone polls it
   pdl_wait();
   const bool weights_ok = mbar_wait(bar, 0, p.status);
-  if (!weights_ok || *reinterpret_cast<volatile int*>(p.status) != 0) return;
+  // A CTA of a split-K cluster never leaves early: its partners read its shared
+  // memory after the cluster barrier. On a raised status it computes a result
+  // the flagged tick discards; every other kernel simply returns.
+  if (EPI != kEpiResidual && (!weights_ok || *reinterpret_cast<volatile int*>(p.status) != 0)) return;
 
   const int n_mtiles = (p.M + kTokTile - 1) / kTokTile;
   const int mt_begin = blockIdx.z * p.m_tiles_per_cta;
@@ -177,16 +188,34 @@ __global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
           *reinterpret_cast<uint32_t*>(p.y + static_cast<size_t>(m0 + m) * p.ldy + nb0 * 16 + n) = v;
         }
       }
-    } else if (EPI == kEpiAtomic) {
-      constexpr int NQ = NT / 4;
-      for (int i = tid; i < NQ * kTokTile; i += kThreads) {
-        const int n = (i % NQ) * 4;
-        const int m = i / NQ;
+    } else if (EPI == kEpiResidual) {
+      // this CTA's split partial -> warp-0 slice of sR, then cluster-wide ordered sum
+      for (int i = tid; i < NT * kTokTile; i += kThreads) {
+        const int n = i / kTokTile;
+        const int m = i - n * kTokTile;
+        sR[static_cast<size_t>(n) * kRedStride + m] = red(n, m);
+      }
+      cg::cluster_group cluster = cg::this_cluster();
+      cluster.sync();
+      const int n_split = static_cast<int>(cluster.num_blocks());
+      const int rank = static_cast<int>(cluster.block_rank());
+      const int rows_per = (kTokTile + n_split - 1) / n_split;
+      const int r0 = rank * rows_per;
+      const int r1 = min(kTokTile, r0 + rows_per);
+      for (int i = tid; i < (r1 - r0) * NT; i += kThreads) {
+        const int m = r0 + i / NT;
+        const int n = i % NT;
         if (m0 + m < p.M) {
-          const float4 v = make_float4(red(n, m), red(n + 1, m), red(n + 2, m), red(n + 3, m));
-          atomicAdd(reinterpret_cast<float4*>(p.xo + static_cast<size_t>(m0 + m) * p.ldxo + nb0 * 16 + n), v);
+          float acc_s = 0.f;
+          for (int s = 0; s < n_split; ++s) {
+            const float* remote = cluster.map_shared_rank(sR, s);
+            acc_s += remote[static_cast<size_t>(n) * kRedStride + m];
+          }
+          float* xo = p.xo + static_cast<size_t>(m0 + m) * p.ldxo + nb0 * 16 + n;
+          *xo = *xo + acc_s;
         }
       }
+      cluster.sync();  // remote reads done before any CTA reuses or releases its shared memory
     } else {  // kEpiSwiglu: block j rows 0..7 = gate of h columns (nb0+j)*8 + r, rows 8..15 = up
       constexpr int NH = NB * 8;
       for (int i = tid; i < NH * kTokTile; i += kThreads) {
@@ -218,8 +247,8 @@ const void* select_kernel(int nb, int pro, int epi) {
   FSX_SEL(2, kProNorm, kEpiStore)
   FSX_SEL(1, kProNorm, kEpiSwiglu)
   FSX_SEL(2, kProNorm, kEpiSwiglu)
-  FSX_SEL(1, kProCopy, kEpiAtomic)
-  FSX_SEL(2, kProCopy, kEpiAtomic)
+  FSX_SEL(1, kProCopy, kEpiResidual)
+  FSX_SEL(2, kProCopy, kEpiResidual)
   FSX_SEL(1, kProCopy, kEpiStore)
   FSX_SEL(2, kProCopy, kEpiStore)
 #undef FSX_SEL
@@ -231,7 +260,7 @@ const void* select_kernel(int nb, int pro, int epi) {
 cudaError_t gemm_set_attributes() {
   const int nbs[2] = {1, 2};
   const int pros[2] = {kProNorm, kProCopy};
-  const int epis[3] = {kEpiStore, kEpiAtomic, kEpiSwiglu};
+  const int epis[3] = {kEpiStore, kEpiResidual, kEpiSwiglu};
   for (int nb : nbs)
     for (int pro : pros)
       for (int epi : epis) {
@@ -249,6 +278,11 @@ GemmPlan plan_gemm(int n_rows, int K, int M, int nb, int ks, int prologue, int e
   pl.ks = ks;
   pl.prologue = prologue;
   pl.epilogue = epilogue;
+  if (epilogue == kEpiResidual) {  // the K splits of a tile form one cluster (portable size <= 8)
+    const int min_ks = (K + 8 * 64 - 1) / (8 * 64) * 64;
+    if (ks < min_ks) ks = min_ks;
+    pl.ks = ks;
+  }
   const int nx = n_rows / (16 * nb);
   const int ny = (K + ks - 1) / ks;
   const int m_tiles = (M + kTokTile - 1) / kTokTile;
@@ -270,21 +304,33 @@ cudaError_t launch_gemm(const GemmPlan& pl, const GemmArgs& args_in, cudaStream_
   const void* fn = select_kernel(pl.nb, pl.prologue, pl.epilogue);
   if (!fn) return cudaErrorInvalidValue;
   void* kargs[] = {&args};
-  return launch_ex(fn, pl.grid, dim3(kThreads), pl.smem, stream, pdl, kargs);
+  const int cluster_y = pl.epilogue == kEpiResidual ? static_cast<int>(pl.grid.y) : 1;
+  return launch_ex(fn, pl.grid, dim3(kThreads), pl.smem, stream, pdl, kargs, cluster_y);
 }
 
 cudaError_t launch_ex(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool pdl,
-                      void** args) {
+                      void** args, int cluster_y) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  int n = 0;
+  if (pdl) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  if (cluster_y > 1) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = 1;
+    attr[n].val.clusterDim.y = static_cast<unsigned>(cluster_y);
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = n;
   return cudaLaunchKernelExC(&cfg, fn, args);
 }
 

@@ -26,7 +26,7 @@ struct TickArgs {
 // ------------------------------------------------------------------ GEMM
 // Y[M, N] = A[M, K] . W[N, K]^T with W packed as 16x16 fp16 fragment blocks.
 enum GemmPrologue { kProNorm = 0, kProCopy = 1 };
-enum GemmEpilogue { kEpiStore = 0, kEpiAtomic = 1, kEpiSwiglu = 2 };
+enum GemmEpilogue { kEpiStore = 0, kEpiResidual = 1, kEpiSwiglu = 2 };
 
 struct GemmArgs {
   const uint4* w;      // packed weights: block (nb, kb) = 32 x uint4 at (nb * K/16 + kb) * 32
@@ -45,7 +45,7 @@ struct GemmArgs {
   // epilogue kEpiStore: y[m, n] fp16; kEpiSwiglu: y[m, n/2] = silu(gate) * up fp16
   __half* y;
   int ldy;
-  // epilogue kEpiAtomic: xo[m, n] += partial (fp32)
+  // epilogue kEpiResidual: xo[m, n] += sum over the K splits (one cluster), fp32
   float* xo;
   int ldxo;
   int* status;
@@ -121,8 +121,8 @@ struct HeadArgs {
 cudaError_t launch_head(const HeadArgs& a, cudaStream_t stream, bool pdl);
 
 // Launch helper: cudaLaunchKernelEx with the programmatic-stream-serialisation
-// attribute when `pdl` is set.
+// attribute when `pdl` is set and a (1, cluster_y, 1) cluster when cluster_y > 1.
 cudaError_t launch_ex(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
-                      bool pdl, void** args);
+                      bool pdl, void** args, int cluster_y = 1);
 
 }  // namespace fsx
