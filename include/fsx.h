@@ -181,6 +181,29 @@ fsx_status fsx_attention(const void* d_q, long long q_stride,
                          int n_splits, void* d_out, float* d_lse,
                          void* d_workspace, size_t workspace_bytes, void* stream);
 
+/* fsx_attention without any scratch argument and without any allocation.
+ * The paper has no counterpart: this entry point exists for callers that may
+ * not allocate device memory once they are running and cannot lend a scratch
+ * buffer either -- e.g. a real-time vehicle stack that reserves all GPU memory
+ * at start-up, because a run-time cudaMalloc can stall on a device-wide
+ * synchronisation or fail under fragmentation, which a 50 ms control tick
+ * cannot absorb. Arguments and results are those of fsx_attention. The
+ * scratch is a 4 MiB array inside the library image, held on every GPU that
+ * loads the library until the process exits; calls for which
+ * fsx_attention_workspace_bytes(B, n_heads, n_q, n_splits) exceeds 4 MiB are
+ * rejected with FSX_ERR_INVALID_ARG before anything is enqueued (n_splits = 1
+ * needs only the status word, for any B). All calls on a device share
+ * that array, so calls whose kernels overlap on the GPU race and must be
+ * serialised by the caller. The first call on each device resolves the array's
+ * device address with that device current; make it before capturing a stream.
+ * Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
+fsx_status fsx_attention_noalloc(const void* d_q, long long q_stride,
+                                 const void* d_k_own, const void* d_v_own, long long own_stride,
+                                 int n_q, int n_own,
+                                 const void* d_k_cache, const void* d_v_cache, int cache_dtype,
+                                 const int64_t* d_offsets, int B, int n_heads, int head_dim,
+                                 int n_splits, void* d_out, float* d_lse, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

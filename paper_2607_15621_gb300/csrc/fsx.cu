@@ -49,6 +49,11 @@ constexpr int kClassQkv = 0, kClassAttn = 1, kClassWo = 2, kClassGateUp = 3, kCl
 
 }  // namespace
 
+namespace fsx {
+// Lets the other translation units of the library report a message through fsx_last_error().
+void set_error_message(const char* msg) { snprintf(g_err, sizeof(g_err), "%s", msg ? msg : ""); }
+}  // namespace fsx
+
 struct fsx_handle_s {
   fsx_config cfg{};
   int device = 0;

@@ -74,6 +74,8 @@ def _load():
         "fsx_attention_workspace_bytes": (ctypes.c_size_t, [i32, i32, i32, i32]),
         "fsx_attention": (i32, [vp, ctypes.c_longlong, vp, vp, ctypes.c_longlong, i32, i32, vp, vp, i32,
                                 vp, i32, i32, i32, i32, vp, vp, vp, ctypes.c_size_t, vp]),
+        "fsx_attention_noalloc": (i32, [vp, ctypes.c_longlong, vp, vp, ctypes.c_longlong, i32, i32, vp, vp,
+                                        i32, vp, i32, i32, i32, i32, vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -95,7 +97,7 @@ def lib():
 def declared_symbols() -> list[str]:
     return ["fsx_create", "fsx_tick", "fsx_tick_host", "fsx_tick_debug", "fsx_get_status", "fsx_last_error",
             "fsx_destroy", "fsx_weight_bytes", "fsx_tick_launches", "fsx_set_kernel_timing",
-            "fsx_kernel_time", "fsx_attention_workspace_bytes", "fsx_attention"]
+            "fsx_kernel_time", "fsx_attention_workspace_bytes", "fsx_attention", "fsx_attention_noalloc"]
 
 
 def last_error() -> str:
@@ -221,4 +223,15 @@ def attention(q, q_stride, k_own, v_own, own_stride, n_q, n_own, k_cache, v_cach
     check(lib().fsx_attention(_ptr(q), q_stride, _ptr(k_own), _ptr(v_own), own_stride, n_q, n_own,
                               _ptr(k_cache), _ptr(v_cache), code, _ptr(offsets), B, n_heads, 128, n_splits,
                               _ptr(out), _ptr(lse), _ptr(workspace), ws_bytes, _stream(stream)))
+    return out
+
+
+def attention_noalloc(q, q_stride, k_own, v_own, own_stride, n_q, n_own, k_cache, v_cache, cache_dtype, offsets,
+                      B, n_heads, n_splits, out, lse, stream=None):
+    """fsx_attention_noalloc through the C ABI: same results as attention(), with the
+    library's static scratch instead of a caller buffer (nothing is allocated)."""
+    code = {"fp32": FSX_F32, "bf16": FSX_BF16}[cache_dtype]
+    check(lib().fsx_attention_noalloc(_ptr(q), q_stride, _ptr(k_own), _ptr(v_own), own_stride, n_q, n_own,
+                                      _ptr(k_cache), _ptr(v_cache), code, _ptr(offsets), B, n_heads, 128,
+                                      n_splits, _ptr(out), _ptr(lse), _stream(stream)))
     return out
