@@ -29,7 +29,7 @@ sys.path.insert(0, ROOT)
 METRIC = "vehicle-ticks/s (1e6 / us-per-tick x B) of the action-expert tick"
 UNIT = "vehicle-ticks/s"
 FALLBACK_HBM_GBS = 6800.0
-KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down"]
+KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down", "persistent"]
 
 
 def parse():
@@ -239,6 +239,8 @@ def main():
 
     # ---- dominant kernel: CUDA events around its launches inside the replayed tick graph
     kclass = args.kernel_class
+    if ex.launches(B) == 1:  # single-launch persistent tick: the tick kernel is the dominant kernel
+        kclass = "persistent"
     ex.set_kernel_timing(True, kclass)
     kt_ms, kt_n = [], 0
     for i in range(max(args.steps // 4, 5) + 2):
@@ -257,7 +259,10 @@ def main():
         "gate_up": 2 * f * d * 2 + M * d * 4 + M * f * 2,
         "down": d * f * 2 + M * f * 2 + 2 * M * d * 4,
         "attention": int(np.sum(lengths)) * 2 * hd * (2 if dtype == "bf16" else 4) + M * 3 * hd * 2 + M * hd * 2,
+        "persistent": None,
     }[kclass]
+    if unit_bytes is None:  # one launch = the whole tick: weights + cache rows
+        unit_bytes = algorithmic_bytes(dims, lengths, dtype, ex.weight_bytes())[0]
     hbm, peak_kind = peaks()
     achieved = unit_bytes / per_launch_s / 1e9
     tick_bytes, kv_bytes = algorithmic_bytes(dims, lengths, dtype, ex.weight_bytes())

@@ -148,9 +148,11 @@ int fsx_tick_launches(fsx_handle h, int B);
 /* Per-kernel-class timing of graph ticks, for roofline reports. With enable=1
  * later fsx_tick calls replay a graph variant that records CUDA events around
  * every launch of kernel class `kclass` (0 = QKV projection, 1 = attention,
- * 2 = output projection, 3 = SwiGLU gate/up, 4 = down projection). fsx_kernel_time
+ * 2 = output projection, 3 = SwiGLU gate/up, 4 = down projection, 5 = persistent
+ * tick). fsx_kernel_time
  * returns the summed event time (ms) and launch count of the most recent tick
- * (synchronises the stream of that tick). */
+ * (synchronises the stream of that tick). Class 5 times the single-launch
+ * persistent tick used for B = 1 (then fsx_tick_launches(h, 1) == 1). */
 fsx_status fsx_set_kernel_timing(fsx_handle h, int enable, int kclass);
 fsx_status fsx_kernel_time(fsx_handle h, float* ms, int* launches);
 

@@ -9,18 +9,26 @@
 // rows, fp16 own rows) with 16-byte cp.async into a double buffer, converted
 // once to fp16 into an XOR-swizzled tile, and consumed by mma.sync m16n8k16
 // (S = Q K^T, then O += P V with P kept in registers) under an online softmax
-// in the log2 domain. With one split the CTA writes the normalised output;
-// otherwise it writes (O / l, m + log2 l) partials and a second kernel merges
-// them: lse = log2 sum_s 2^lse_s, o = sum_s 2^(lse_s - lse) o_s.
+// in the log2 domain. With one split the CTA writes the normalised output.
+// With 2..8 splits the splits of one (vehicle, head) form a thread-block
+// cluster: each CTA leaves (O / l, m + log2 l) in its shared memory and, after
+// a cluster barrier, merges a slice of the query rows over all splits through
+// distributed shared memory (lse = log2 sum_s 2^lse_s, o = sum_s
+// 2^(lse_s - lse) o_s), in split order. More splits fall back to global
+// partials merged by a second kernel.
+#include <cooperative_groups.h>
 #include <math_constants.h>
 
 #include "device_util.cuh"
 #include "kernels.h"
 
+namespace cg = cooperative_groups;
+
 namespace fsx {
 
 namespace {
 
+constexpr int kMaxClusterSplits = 8;
 constexpr int kWarps = 3;
 constexpr int kThreads = kWarps * 32;
 constexpr int kChunk = 64;
@@ -66,7 +74,7 @@ __device__ __forceinline__ void convert_unit<float>(const unsigned char* raw, ui
   }
 }
 
-template <typename CT>
+template <typename CT, bool CM>
 __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p) {
   extern __shared__ __align__(128) unsigned char smem[];
   constexpr int RB = CacheRow<CT>::kBytes;
@@ -85,7 +93,9 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
 
   pdl_launch_dependents();
   pdl_wait();
-  if (*reinterpret_cast<volatile int*>(p.status) != 0) return;
+  // The CTAs of a merge cluster read each other's shared memory, so they must
+  // all stay; a raised status is honoured per vehicle below instead.
+  if (!CM && *reinterpret_cast<volatile int*>(p.status) != 0) return;
 
   const CT* kc;
   const CT* vc;
@@ -114,7 +124,8 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
   // output slots
   const size_t part_base = (static_cast<size_t>(b) * H + h) * p.n_splits + split;  // partial index
 
-  if (kend <= kbeg) {  // an empty key range contributes nothing
+  const bool empty_range = kend <= kbeg;
+  if (empty_range && !CM) {  // an empty key range contributes nothing
     if (p.n_splits > 1) {
       for (int i = tid; i < kTokTile; i += kThreads) p.part_lse[part_base * kTokTile + i] = -CUDART_INF_F;
       float* po = p.part_o + part_base * kTokTile * kD;
@@ -188,8 +199,8 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
   float l_run[2] = {0.f, 0.f};
   const float scale_log2 = 1.4426950408889634f * rsqrtf(static_cast<float>(kD));
 
-  const int n_chunks = static_cast<int>((kend - kbeg + kChunk - 1) / kChunk);
-  issue_chunk(0, 0);
+  const int n_chunks = empty_range ? 0 : static_cast<int>((kend - kbeg + kChunk - 1) / kChunk);
+  if (n_chunks > 0) issue_chunk(0, 0);
   if (n_chunks > 1) issue_chunk(1, 1);
 
   for (int c = 0; c < n_chunks; ++c) {
@@ -311,8 +322,70 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
   }
 
   // ---- write out
-  const float inv0 = 1.f / l_run[0];
-  const float inv1 = 1.f / l_run[1];
+  const float inv0 = l_run[0] > 0.f ? 1.f / l_run[0] : 0.f;
+  const float inv1 = l_run[1] > 0.f ? 1.f / l_run[1] : 0.f;
+  if (CM) {
+    // Merge of the cluster's splits: after every split finished its key range,
+    // each CTA pushes the rows another rank owns, with its log-sum-exp, into
+    // that rank's (now idle) K/V tile memory; one more barrier; then each
+    // owner merges its rows locally in split order.
+    cg::cluster_group cluster = cg::this_cluster();
+    const int S = static_cast<int>(cluster.num_blocks());
+    const int rank = static_cast<int>(cluster.block_rank());
+    const int rows_per = (kTokTile + S - 1) / S;
+    float* rPo = reinterpret_cast<float*>(tile);            // [S][rows_per][kD]
+    float* rLse = rPo + static_cast<size_t>(S) * rows_per * kD;  // [S][rows_per]
+    cluster.sync();  // every split is done with its tiles
+    {
+      const int own0 = qr0 / rows_per, own1 = qr1 / rows_per;
+      float* d0 = cluster.map_shared_rank(rPo, own0) + (static_cast<size_t>(rank) * rows_per + (qr0 - own0 * rows_per)) * kD;
+      float* d1 = cluster.map_shared_rank(rPo, own1) + (static_cast<size_t>(rank) * rows_per + (qr1 - own1 * rows_per)) * kD;
+#pragma unroll
+      for (int n = 0; n < 16; ++n) {
+        const int d = n * 8 + 2 * (lane & 3);
+        *reinterpret_cast<float2*>(d0 + d) = make_float2(o_acc[n][0] * inv0, o_acc[n][1] * inv0);
+        *reinterpret_cast<float2*>(d1 + d) = make_float2(o_acc[n][2] * inv1, o_acc[n][3] * inv1);
+      }
+      if ((lane & 3) == 0) {
+        cluster.map_shared_rank(rLse, own0)[rank * rows_per + (qr0 - own0 * rows_per)] =
+            l_run[0] > 0.f ? m_run[0] + log2f(l_run[0]) : -CUDART_INF_F;
+        cluster.map_shared_rank(rLse, own1)[rank * rows_per + (qr1 - own1 * rows_per)] =
+            l_run[1] > 0.f ? m_run[1] + log2f(l_run[1]) : -CUDART_INF_F;
+      }
+    }
+    cluster.sync();  // all pushes landed
+    const int q_lo = rank * rows_per;
+    const int q_hi = min(p.n_q, q_lo + rows_per);
+    for (int i = tid; i < (q_hi - q_lo) * (kD / 4); i += kThreads) {
+      const int qq = i / (kD / 4);
+      const int q = q_lo + qq;
+      const int d = (i % (kD / 4)) * 4;
+      float mmax = -CUDART_INF_F;
+      for (int r = 0; r < S; ++r) mmax = fmaxf(mmax, rLse[r * rows_per + qq]);
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      float wsum = 0.f;
+      if (mmax != -CUDART_INF_F) {
+        for (int r = 0; r < S; ++r) {
+          const float w = exp2f(rLse[r * rows_per + qq] - mmax);
+          const float4 v = *reinterpret_cast<const float4*>(rPo + (static_cast<size_t>(r) * rows_per + qq) * kD + d);
+          wsum += w;
+          acc.x += w * v.x;
+          acc.y += w * v.y;
+          acc.z += w * v.z;
+          acc.w += w * v.w;
+        }
+      }
+      const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+      uint2 packed;
+      packed.x = pack_half2(acc.x * inv, acc.y * inv);
+      packed.y = pack_half2(acc.z * inv, acc.w * inv);
+      *reinterpret_cast<uint2*>(p.out + (static_cast<size_t>(b) * p.n_q + q) * p.out_stride + h * kD + d) = packed;
+      if (p.lse != nullptr && d == 0)
+        p.lse[(static_cast<size_t>(b) * H + h) * p.n_q + q] =
+            wsum > 0.f ? (mmax + log2f(wsum)) * 0.6931471805599453f : -CUDART_INF_F;
+    }
+    return;
+  }
   if (p.n_splits == 1) {
     const bool v0 = qr0 < p.n_q;
     const bool v1 = qr1 < p.n_q;
@@ -381,36 +454,45 @@ __global__ void __launch_bounds__(kD) attn_combine_kernel(const AttnArgs p) {
 }  // namespace
 
 size_t attention_workspace_bytes(int B, int n_heads, int n_splits) {
-  if (n_splits <= 1) return 0;
+  if (n_splits <= kMaxClusterSplits) return 0;  // one split writes directly, up to 8 merge in a cluster
   const size_t parts = static_cast<size_t>(B) * n_heads * n_splits;
   return parts * kTokTile * kD * sizeof(float) + parts * kTokTile * sizeof(float);
 }
 
-int attention_launch_count(int n_splits) { return n_splits > 1 ? 2 : 1; }
+int attention_launch_count(int n_splits) { return n_splits > kMaxClusterSplits ? 2 : 1; }
 
 cudaError_t attention_set_attributes() {
-  cudaError_t e = cudaFuncSetAttribute(reinterpret_cast<const void*>(&attn_splitkv_kernel<__nv_bfloat16>),
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(attn_smem_bytes<__nv_bfloat16>()));
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(reinterpret_cast<const void*>(&attn_splitkv_kernel<float>),
-                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(attn_smem_bytes<float>()));
+  const void* fns[4] = {reinterpret_cast<const void*>(&attn_splitkv_kernel<__nv_bfloat16, false>),
+                        reinterpret_cast<const void*>(&attn_splitkv_kernel<__nv_bfloat16, true>),
+                        reinterpret_cast<const void*>(&attn_splitkv_kernel<float, false>),
+                        reinterpret_cast<const void*>(&attn_splitkv_kernel<float, true>)};
+  const size_t bytes[4] = {attn_smem_bytes<__nv_bfloat16>(), attn_smem_bytes<__nv_bfloat16>(),
+                           attn_smem_bytes<float>(), attn_smem_bytes<float>()};
+  for (int i = 0; i < 4; ++i) {
+    cudaError_t e = cudaFuncSetAttribute(fns[i], cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes[i]));
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_attention(const AttnArgs& a_in, int B, int cache_dtype, cudaStream_t stream, bool pdl) {
   AttnArgs a = a_in;
   void* kargs[] = {&a};
   const dim3 grid(a.n_splits, a.n_heads, B);
-  cudaError_t e;
+  const bool cm = a.n_splits > 1 && a.n_splits <= kMaxClusterSplits;
+  const void* fn;
+  size_t smem;
   if (cache_dtype == 1) {
-    e = launch_ex(reinterpret_cast<const void*>(&attn_splitkv_kernel<__nv_bfloat16>), grid, dim3(kThreads),
-                  attn_smem_bytes<__nv_bfloat16>(), stream, pdl, kargs);
+    fn = cm ? reinterpret_cast<const void*>(&attn_splitkv_kernel<__nv_bfloat16, true>)
+            : reinterpret_cast<const void*>(&attn_splitkv_kernel<__nv_bfloat16, false>);
+    smem = attn_smem_bytes<__nv_bfloat16>();
   } else {
-    e = launch_ex(reinterpret_cast<const void*>(&attn_splitkv_kernel<float>), grid, dim3(kThreads),
-                  attn_smem_bytes<float>(), stream, pdl, kargs);
+    fn = cm ? reinterpret_cast<const void*>(&attn_splitkv_kernel<float, true>)
+            : reinterpret_cast<const void*>(&attn_splitkv_kernel<float, false>);
+    smem = attn_smem_bytes<float>();
   }
-  if (e != cudaSuccess || a.n_splits <= 1) return e;
+  cudaError_t e = launch_ex(fn, grid, dim3(kThreads), smem, stream, pdl, kargs, 1, cm ? a.n_splits : 1);
+  if (e != cudaSuccess || a.n_splits <= kMaxClusterSplits) return e;
   return launch_ex(reinterpret_cast<const void*>(&attn_combine_kernel), dim3(a.n_heads, B), dim3(kD), 0, stream,
                    pdl, kargs);
 }

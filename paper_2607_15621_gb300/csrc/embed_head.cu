@@ -40,7 +40,9 @@ __global__ void embed_kernel(const EmbedArgs a) {
         v = static_cast<const float*>(a.targs->frames)[idx];
       }
     }
-    xr[c] = v + pos[c];
+    const float xv = v + pos[c];
+    xr[c] = xv;
+    a.x16[static_cast<size_t>(row) * a.d + c] = __float2half_rn(xv);
   }
 }
 

@@ -23,6 +23,7 @@
 
 #include "../../include/fsx.h"
 #include "kernels.h"
+#include "persistent.h"
 
 using fsx::TickArgs;
 
@@ -45,7 +46,7 @@ fsx_status fail(fsx_status s, const char* fmt, ...) {
                                        __FILE__, __LINE__);                                         \
   } while (0)
 
-constexpr int kClassQkv = 0, kClassAttn = 1, kClassWo = 2, kClassGateUp = 3, kClassDown = 4;
+constexpr int kClassQkv = 0, kClassAttn = 1, kClassWo = 2, kClassGateUp = 3, kClassDown = 4, kClassPersistent = 5;
 
 }  // namespace
 
@@ -70,6 +71,7 @@ struct fsx_handle_s {
   float *final_norm = nullptr, *head_w = nullptr, *head_b = nullptr;
   // workspace
   float* x = nullptr;
+  __half* x16 = nullptr;
   __half* qkv = nullptr;
   __half* o = nullptr;
   __half* hbuf = nullptr;
@@ -79,6 +81,12 @@ struct fsx_handle_s {
   TickArgs* d_args = nullptr;
   TickArgs h_args{};
   bool args_valid = false;
+  // persistent single-vehicle tick
+  bool persist_ok = false;
+  void* p_arena = nullptr;
+  long long p_layer_bytes = 0, p_a_cta = 0, p_b_offset = 0, p_b_cta = 0;
+  float* p_x = nullptr;
+  int* p_counters = nullptr;
   // host-buffer tick staging
   int64_t* st_offsets = nullptr;
   void* st_frames = nullptr;
@@ -103,7 +111,7 @@ namespace {
 int attention_splits(const fsx_handle_s* h, int B) {
   const int work = B * h->cfg.n_heads;
   int s = (2 * h->sm_count) / std::max(work, 1);
-  return std::min(std::max(s, 1), 16);
+  return std::min(std::max(s, 1), 8);  // <= 8: the splits merge inside one thread-block cluster
 }
 
 fsx_status check_config(const fsx_config* c) {
@@ -130,7 +138,7 @@ fsx_status check_config(const fsx_config* c) {
 // block (nb, kb) holds, for lane l, rows r = 16nb + l/4 and r + 8 and columns
 // c = 16kb + 2(l%4) (+1, +8, +9) in register order a0..a7.
 template <typename RowFn>
-void pack_fragments(RowFn row, int N, int K, __half* out) {
+void pack_fragments(RowFn row, int N, int K, __half* out, const float* col_scale = nullptr) {
   const int kbs = K / 16;
   for (int nb = 0; nb < N / 16; ++nb) {
     for (int lane = 0; lane < 32; ++lane) {
@@ -140,20 +148,27 @@ void pack_fragments(RowFn row, int N, int K, __half* out) {
       for (int kb = 0; kb < kbs; ++kb) {
         __half* o = out + ((static_cast<size_t>(nb) * kbs + kb) * 32 + lane) * 8;
         const int k = kb * 16 + c;
-        o[0] = __float2half_rn(r0[k]);
-        o[1] = __float2half_rn(r0[k + 1]);
-        o[2] = __float2half_rn(r1[k]);
-        o[3] = __float2half_rn(r1[k + 1]);
-        o[4] = __float2half_rn(r0[k + 8]);
-        o[5] = __float2half_rn(r0[k + 9]);
-        o[6] = __float2half_rn(r1[k + 8]);
-        o[7] = __float2half_rn(r1[k + 9]);
+        auto sc = [&](int kk) { return col_scale ? col_scale[kk] : 1.f; };
+        o[0] = __float2half_rn(r0[k] * sc(k));
+        o[1] = __float2half_rn(r0[k + 1] * sc(k + 1));
+        o[2] = __float2half_rn(r1[k] * sc(k));
+        o[3] = __float2half_rn(r1[k + 1] * sc(k + 1));
+        o[4] = __float2half_rn(r0[k + 8] * sc(k + 8));
+        o[5] = __float2half_rn(r0[k + 9] * sc(k + 9));
+        o[6] = __float2half_rn(r1[k + 8] * sc(k + 8));
+        o[7] = __float2half_rn(r1[k + 9] * sc(k + 9));
       }
     }
   }
 }
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+bool use_persistent(const fsx_handle_s* h, int B) {
+  if (B != 1 || !h->persist_ok) return false;
+  const char* off = std::getenv("FSX_DISABLE_PERSISTENT");
+  return !(off && off[0] == '1');
+}
 
 fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_capture, bool timed) {
   const fsx_config& c = h->cfg;
@@ -168,6 +183,41 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     return cudaEventRecordWithFlags(ev, st, cudaEventRecordExternal);
   };
 
+  if (use_persistent(h, B)) {
+    fsx::PersistArgs pa{};
+    pa.warena = static_cast<const unsigned char*>(h->p_arena);
+    pa.layer_bytes = h->p_layer_bytes;
+    pa.a_cta_bytes = h->p_a_cta;
+    pa.b_offset = h->p_b_offset;
+    pa.b_cta_bytes = h->p_b_cta;
+    pa.act_emb = h->act_emb;
+    pa.pos_emb = h->pos_emb;
+    pa.final_norm = h->final_norm;
+    pa.head_w = h->head_w;
+    pa.head_b = h->head_b;
+    pa.targs = h->d_args;
+    pa.n_layers = c.n_layers;
+    pa.d = d;
+    pa.H = c.n_heads;
+    pa.F = F;
+    pa.n_action = c.n_action;
+    pa.n_frame = c.n_frame;
+    pa.n_waypoints = c.n_waypoints;
+    pa.n_b_clusters = F / 64;
+    pa.frame_dtype = c.frame_dtype;
+    pa.max_total = c.max_total_cache_tokens;
+    pa.X = h->p_x;
+    pa.counters = h->p_counters;
+    pa.status = h->status;
+    pa.attn_capture = attn_capture;
+    FSX_CUDA(cudaMemsetAsync(h->p_counters, 0, sizeof(int) * (2 * c.n_layers + 1), st));
+    FSX_CUDA(mark(kClassPersistent, true));
+    FSX_CUDA(fsx::launch_persistent(pa, c.cache_dtype, st));
+    FSX_CUDA(mark(kClassPersistent, false));
+    if (timed) h->timed_pairs = pair;
+    return FSX_OK;
+  }
+
   fsx::EmbedArgs ea{};
   ea.act_emb = h->act_emb;
   ea.pos_emb = h->pos_emb;
@@ -179,10 +229,12 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
   ea.B = B;
   ea.max_total = c.max_total_cache_tokens;
   ea.x = h->x;
+  ea.x16 = h->x16;
   ea.status = h->status;
   FSX_CUDA(fsx::launch_embed(ea, st, pdl));
 
-  const fsx::GemmPlan pq = fsx::plan_gemm(3 * HD, d, M, 2, d, fsx::kProNorm, fsx::kEpiStore, h->sm_count);
+  // 48-row QKV tiles: 256 CTAs at two per SM run as one wave
+  const fsx::GemmPlan pq = fsx::plan_gemm(3 * HD, d, M, 3, d, fsx::kProNorm, fsx::kEpiStore, h->sm_count);
   const fsx::GemmPlan po = fsx::plan_gemm(d, HD, M, 2, 512, fsx::kProCopy, fsx::kEpiResidual, h->sm_count);
   const fsx::GemmPlan pg = fsx::plan_gemm(2 * F, d, M, 1, d, fsx::kProNorm, fsx::kEpiSwiglu, h->sm_count);
   const fsx::GemmPlan pd = fsx::plan_gemm(d, F, M, 1, 256, fsx::kProCopy, fsx::kEpiResidual, h->sm_count);
@@ -196,9 +248,8 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     g.w = h->w_qkv[l];
     g.n_rows = 3 * HD;
     g.K = d;
-    g.x = h->x;
-    g.gamma = h->attn_norm + static_cast<size_t>(l) * d;
-    g.ldx = d;
+    g.x16 = h->x16;
+    g.ldx16 = d;
     g.y = h->qkv;
     g.ldy = 3 * HD;
     FSX_CUDA(mark(kClassQkv, true));
@@ -243,6 +294,7 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     go.a = h->o;
     go.lda = HD;
     go.xo = h->x;
+    go.xo16 = h->x16;
     go.ldxo = d;
     FSX_CUDA(mark(kClassWo, true));
     FSX_CUDA(fsx::launch_gemm(po, go, st, pdl));
@@ -255,9 +307,8 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     gg.w = h->w_gu[l];
     gg.n_rows = 2 * F;
     gg.K = d;
-    gg.x = h->x;
-    gg.gamma = h->mlp_norm + static_cast<size_t>(l) * d;
-    gg.ldx = d;
+    gg.x16 = h->x16;
+    gg.ldx16 = d;
     gg.y = h->hbuf;
     gg.ldy = F;
     FSX_CUDA(mark(kClassGateUp, true));
@@ -274,6 +325,7 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     gd.a = h->hbuf;
     gd.lda = F;
     gd.xo = h->x;
+    gd.xo16 = h->x16;
     gd.ldxo = d;
     FSX_CUDA(mark(kClassDown, true));
     FSX_CUDA(fsx::launch_gemm(pd, gd, st, pdl));
@@ -371,7 +423,7 @@ void free_handle(fsx_handle_s* h) {
   for (cudaEvent_t e : h->tev) cudaEventDestroy(e);
   if (h->last_tick) cudaEventDestroy(h->last_tick);
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
-  void* bufs[] = {h->w_arena, h->params, h->x, h->qkv, h->o, h->hbuf, h->part, h->status, h->d_args,
+  void* bufs[] = {h->p_arena, h->p_x, h->p_counters, h->w_arena, h->params, h->x, h->x16, h->qkv, h->o, h->hbuf, h->part, h->status, h->d_args,
                   h->st_offsets, h->st_frames, h->st_waypoints};
   for (void* p : bufs)
     if (p) cudaFree(p);
@@ -448,7 +500,7 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
             if (r < 2 * HD) return wk + static_cast<size_t>(r - HD) * d;
             return wv + static_cast<size_t>(r - 2 * HD) * d;
           },
-          3 * HD, d, reinterpret_cast<__half*>(base));
+          3 * HD, d, reinterpret_cast<__half*>(base), w->attn_norm + static_cast<size_t>(l) * d);
       const float* wo = w->wo + hd_d * l;
       pack_fragments([&](int r) -> const float* { return wo + static_cast<size_t>(r) * HD; }, d, HD,
                      reinterpret_cast<__half*>(base + b_qkv));
@@ -460,7 +512,7 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
             const int blk = p >> 4, r = p & 15;
             return r < 8 ? wg + static_cast<size_t>(blk * 8 + r) * d : wu + static_cast<size_t>(blk * 8 + r - 8) * d;
           },
-          2 * F, d, reinterpret_cast<__half*>(base + b_qkv + b_o));
+          2 * F, d, reinterpret_cast<__half*>(base + b_qkv + b_o), w->mlp_norm + static_cast<size_t>(l) * d);
       const float* wd = w->w_down + static_cast<size_t>(d) * F * l;
       pack_fragments([&](int r) -> const float* { return wd + static_cast<size_t>(r) * F; }, d, F,
                      reinterpret_cast<__half*>(base + b_qkv + b_o + b_gu));
@@ -480,6 +532,81 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
     h->w_o.push_back(reinterpret_cast<const uint4*>(base + b_qkv));
     h->w_gu.push_back(reinterpret_cast<const uint4*>(base + b_qkv + b_o));
     h->w_dn.push_back(reinterpret_cast<const uint4*>(base + b_qkv + b_o + b_gu));
+  }
+
+  // ---- stream-ordered weights of the persistent single-vehicle tick
+  {
+    const int H = cfg->n_heads;
+    const int n_b = F / 64;
+    int max_clusters = 0;
+    const bool shape_ok = d == 512 && T <= fsx::kTokTile && F % 64 == 0 && n_b <= H &&
+                          H * fsx::kPersistCluster <= h->sm_count && std::getenv("FSX_NO_PERSISTENT_BUILD") == nullptr;
+    if (shape_ok && fsx::persistent_set_attributes(d) == cudaSuccess)
+      max_clusters = fsx::persistent_max_clusters(d, cfg->cache_dtype);
+    cudaGetLastError();
+    if (shape_ok && max_clusters >= H) {
+      const int G = H * fsx::kPersistCluster;
+      const long long chunk = fsx::kPersistChunk;
+      h->p_a_cta = chunk * fsx::kPersistAChunks;
+      h->p_b_cta = chunk * fsx::kPersistBChunks;
+      h->p_b_offset = h->p_a_cta * G;
+      h->p_layer_bytes = h->p_b_offset + h->p_b_cta * n_b * fsx::kPersistCluster;
+      const size_t total = static_cast<size_t>(h->p_layer_bytes) * L;
+      FSX_CUDA_H(cudaMalloc(&h->p_arena, total));
+      std::vector<__half> host(total / 2);
+      const size_t hd_d = static_cast<size_t>(HD) * d;
+      auto pack_layer = [&](int l) {
+        unsigned char* base = reinterpret_cast<unsigned char*>(host.data()) + static_cast<size_t>(h->p_layer_bytes) * l;
+        const float* g1 = w->attn_norm + static_cast<size_t>(l) * d;
+        const float* g2 = w->mlp_norm + static_cast<size_t>(l) * d;
+        for (int cta = 0; cta < G; ++cta) {
+          const int head = cta / fsx::kPersistCluster, rank = cta % fsx::kPersistCluster;
+          unsigned char* a = base + static_cast<size_t>(cta) * h->p_a_cta;
+          const float* mats[3] = {w->wq + hd_d * l, w->wk + hd_d * l, w->wv + hd_d * l};
+          for (int i = 0; i < 6; ++i) {  // q, q, k, k, v, v: 16 head dims each
+            const float* m = mats[i / 2];
+            const int dim0 = head * fsx::kHeadDim + rank * 32 + (i % 2) * 16;
+            pack_fragments([&](int r) -> const float* { return m + static_cast<size_t>(dim0 + r) * d; }, 16, d,
+                           reinterpret_cast<__half*>(a + i * chunk), g1);
+          }
+          const float* wo = w->wo + hd_d * l;
+          for (int i = 0; i < 2; ++i) {  // 64 output columns x this head's 128 inputs
+            const int col0 = rank * 128 + i * 64;
+            pack_fragments([&](int r) -> const float* {
+              return wo + static_cast<size_t>(col0 + r) * HD + head * fsx::kHeadDim;
+            }, 64, fsx::kHeadDim, reinterpret_cast<__half*>(a + (6 + i) * chunk));
+          }
+        }
+        const float* wg = w->w_gate + static_cast<size_t>(F) * d * l;
+        const float* wu = w->w_up + static_cast<size_t>(F) * d * l;
+        const float* wd = w->w_down + static_cast<size_t>(d) * F * l;
+        for (int cta = 0; cta < n_b * fsx::kPersistCluster; ++cta) {
+          const int cl = cta / fsx::kPersistCluster, rank = cta % fsx::kPersistCluster;
+          unsigned char* b = base + h->p_b_offset + static_cast<size_t>(cta) * h->p_b_cta;
+          for (int j = 0; j < 2; ++j) {  // 8 gate rows then the matching 8 up rows
+            const int hc0 = cl * 64 + rank * 16 + j * 8;
+            pack_fragments([&](int r) -> const float* {
+              return r < 8 ? wg + static_cast<size_t>(hc0 + r) * d : wu + static_cast<size_t>(hc0 + r - 8) * d;
+            }, 16, d, reinterpret_cast<__half*>(b + j * chunk), g2);
+          }
+          pack_fragments([&](int r) -> const float* {  // 128 output columns x this cluster's 64 SwiGLU inputs
+            return wd + static_cast<size_t>(rank * 128 + r) * F + cl * 64;
+          }, 128, 64, reinterpret_cast<__half*>(b + 2 * chunk));
+        }
+      };
+      const int n_threads = std::max(1, std::min<int>(16, static_cast<int>(std::thread::hardware_concurrency())));
+      std::vector<std::thread> pool;
+      for (int t = 0; t < n_threads; ++t)
+        pool.emplace_back([&, t]() {
+          for (int l = t; l < L; l += n_threads) pack_layer(l);
+        });
+      for (auto& th : pool) th.join();
+      FSX_CUDA_H(cudaMemcpy(h->p_arena, host.data(), total, cudaMemcpyHostToDevice));
+      FSX_CUDA_H(cudaMalloc(&h->p_x, static_cast<size_t>(3) * fsx::kTokTile * d * sizeof(float)));
+      FSX_CUDA_H(cudaMemset(h->p_x, 0, static_cast<size_t>(3) * fsx::kTokTile * d * sizeof(float)));
+      FSX_CUDA_H(cudaMalloc(&h->p_counters, sizeof(int) * (2 * L + 1)));
+      h->persist_ok = true;
+    }
   }
 
   // ---- fp32 parameters
@@ -510,6 +637,7 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
   const size_t Mmax = static_cast<size_t>(cfg->max_batch) * T;
   const size_t m_pad = (Mmax + fsx::kTokTile - 1) / fsx::kTokTile * fsx::kTokTile;
   FSX_CUDA_H(cudaMalloc(&h->x, m_pad * d * sizeof(float)));
+  FSX_CUDA_H(cudaMalloc(&h->x16, m_pad * d * sizeof(__half)));
   FSX_CUDA_H(cudaMalloc(&h->qkv, m_pad * 3 * HD * sizeof(__half)));
   FSX_CUDA_H(cudaMalloc(&h->o, m_pad * HD * sizeof(__half)));
   FSX_CUDA_H(cudaMalloc(&h->hbuf, m_pad * F * sizeof(__half)));
@@ -607,12 +735,13 @@ long long fsx_weight_bytes(fsx_handle h) { return h ? h->weight_bytes : 0; }
 
 int fsx_tick_launches(fsx_handle h, int B) {
   if (!h || B < 1) return 0;
+  if (use_persistent(h, B)) return 1;
   return 2 + h->cfg.n_layers * (4 + fsx::attention_launch_count(attention_splits(h, B)));
 }
 
 fsx_status fsx_set_kernel_timing(fsx_handle h, int enable, int kclass) {
   if (!h) return fail(FSX_ERR_INVALID_ARG, "handle is NULL");
-  if (kclass < kClassQkv || kclass > kClassDown) return fail(FSX_ERR_INVALID_ARG, "kernel class %d unknown", kclass);
+  if (kclass < kClassQkv || kclass > kClassPersistent) return fail(FSX_ERR_INVALID_ARG, "kernel class %d unknown", kclass);
   std::lock_guard<std::mutex> lock(h->mu);
   if (enable && kclass != h->timing_class) {
     for (auto& kv : h->timed_graphs) cudaGraphExecDestroy(kv.second);

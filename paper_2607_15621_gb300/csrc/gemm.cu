@@ -9,8 +9,11 @@
 // contiguous run of fragment-ordered blocks that one thread fetches with bulk
 // copies (mbarrier completion) BEFORE waiting on the previous kernel, so the
 // weight stream overlaps the tail of the preceding step. The activation tile
-// (48 x K range, fp16) is staged in shared memory by the prologue, either as
-// RMSNorm(x) * gamma from the fp32 residual stream or as a copy of fp16 rows.
+// (48 x K range, fp16) arrives by per-row bulk copies on a second mbarrier:
+// for the RMSNorm-fused projections it is the fp16 copy of the residual
+// stream (the norm gain is folded into the packed weights and the per-row
+// 1/rms, computed from the staged tile, scales the accumulators), otherwise
+// the fp16 input rows (attention output, SwiGLU activations).
 // Warps split the K range; a shared-memory reduction combines them and the
 // epilogue stores fp16, applies the SwiGLU gate to row pairs packed next to
 // each other, or adds the split-K sum into the fp32 residual stream. The K
@@ -34,9 +37,19 @@ constexpr int kRedStride = kTokTile + 4;
 
 __host__ __device__ constexpr int a_stride(int ks) { return ks + 8; }  // halves, 16-byte row pad
 
-__host__ __device__ inline size_t gemm_smem_bytes(int nb, int ks) {
-  return 128 + static_cast<size_t>(nb) * (ks / 16) * 512 + static_cast<size_t>(kTokTile) * a_stride(ks) * 2 +
-         static_cast<size_t>(4) * (16 * nb) * kRedStride * 4;
+// Shared memory: [256 B barriers + 1/rms][weights][activation tile, reused as
+// the cross-warp reduction buffer after the MMAs][split-K receive buffer].
+constexpr int kRecvRows = kTokTile + 8;  // >= n_split * ceil(48 / n_split) for n_split <= 8
+
+__host__ __device__ inline size_t gemm_a_region(int nb, int ks) {
+  const size_t a = static_cast<size_t>(kTokTile) * a_stride(ks) * 2;
+  const size_t r = static_cast<size_t>(4) * (16 * nb) * kRedStride * 4;
+  return a > r ? a : r;
+}
+
+__host__ __device__ inline size_t gemm_smem_bytes(int nb, int ks, int epi) {
+  return 256 + static_cast<size_t>(nb) * (ks / 16) * 512 + gemm_a_region(nb, ks) +
+         (epi == kEpiResidual ? static_cast<size_t>(kRecvRows) * (16 * nb) * 4 : 0);
 }
 
 template <int NB, int PRO, int EPI>
@@ -45,10 +58,13 @@ __global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
   extern __shared__ __align__(128) unsigned char smem[];
   const int ks = p.ks;
   const int lda_s = a_stride(ks);
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem);
-  uint4* sW = reinterpret_cast<uint4*>(smem + 128);
-  __half* sA = reinterpret_cast<__half*>(smem + 128 + static_cast<size_t>(NB) * (ks / 16) * 512);
-  float* sR = reinterpret_cast<float*>(sA + static_cast<size_t>(kTokTile) * lda_s);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem);       // weights
+  uint64_t* act_bar = bar + 1;                              // activation tile
+  float* s_rstd = reinterpret_cast<float*>(smem + 16);     // [48] per-row 1/rms (kProNorm)
+  uint4* sW = reinterpret_cast<uint4*>(smem + 256);
+  __half* sA = reinterpret_cast<__half*>(smem + 256 + static_cast<size_t>(NB) * (ks / 16) * 512);
+  float* sR = reinterpret_cast<float*>(sA);  // reused once every warp finished its MMAs
+  float* recv = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sA) + gemm_a_region(NB, ks));
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
@@ -61,6 +77,7 @@ __global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
   pdl_launch_dependents();
   if (tid == 0) {
     mbar_init(bar, 1);
+    mbar_init(act_bar, 1);
     mbar_arrive_expect_tx(bar, static_cast<uint32_t>(NB * (kl / 16) * 512));
 #pragma unroll
     for (int j = 0; j < NB; ++j) {
@@ -68,7 +85,7 @@ __global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
       bulk_g2s(sW + static_cast<size_t>(j) * (ks / 16) * 32, src, static_cast<uint32_t>((kl / 16) * 512), bar);
     }
   }
-  __syncthreads();  // barrier initialised before anyone polls it
+  __syncthreads();  // barriers initialised before anyone polls them
   pdl_wait();
   const bool weights_ok = mbar_wait(bar, 0, p.status);
   // A CTA of a split-K cluster never leaves early: its partners read its shared
@@ -79,50 +96,42 @@ __global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
   const int n_mtiles = (p.M + kTokTile - 1) / kTokTile;
   const int mt_begin = blockIdx.z * p.m_tiles_per_cta;
   const int mt_end = min(n_mtiles, mt_begin + p.m_tiles_per_cta);
+  const __half* a_src = PRO == kProNorm ? p.x16 : p.a;
+  const int a_ld = PRO == kProNorm ? p.ldx16 : p.lda;
 
   for (int mt = mt_begin; mt < mt_end; ++mt) {
     const int m0 = mt * kTokTile;
-    // ---------------- prologue: activation tile -> sA (fp16)
-    if (PRO == kProNorm) {
+    const int rows = min(kTokTile, p.M - m0);
+    // ---------------- prologue: activation rows -> sA by bulk copies, padding rows zeroed
+    if (warp == 0) {
+      if (lane == 0) mbar_arrive_expect_tx(act_bar, static_cast<uint32_t>(rows * kl * 2));
+      __syncwarp();
+      for (int r = lane; r < rows; r += 32)
+        bulk_g2s(sA + static_cast<size_t>(r) * lda_s, a_src + static_cast<size_t>(m0 + r) * a_ld + k0,
+                 static_cast<uint32_t>(kl * 2), act_bar);
+    }
+    for (int i = tid; i < (kTokTile - rows) * (kl / 8); i += kThreads) {
+      const int r = rows + i / (kl / 8);
+      const int c = (i % (kl / 8)) * 8;
+      *reinterpret_cast<uint4*>(sA + static_cast<size_t>(r) * lda_s + c) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    mbar_wait(act_bar, static_cast<uint32_t>((mt - mt_begin) & 1), p.status);
+    if (PRO == kProNorm) {  // 1/rms of each staged row (the whole row: ks == K)
       for (int r = warp; r < kTokTile; r += 4) {
-        const int m = m0 + r;
-        __half* dst = sA + static_cast<size_t>(r) * lda_s;
-        if (m < p.M) {
-          const float* xr = p.x + static_cast<size_t>(m) * p.ldx;
-          float ss = 0.f;
-          for (int c = lane * 4; c < p.K; c += 128) {
-            const float4 v = *reinterpret_cast<const float4*>(xr + c);
-            ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+        const __half* row = sA + static_cast<size_t>(r) * lda_s;
+        float ss = 0.f;
+        for (int c = lane * 8; c < kl; c += 256) {
+          const uint4 u = *reinterpret_cast<const uint4*>(row + c);
+          const __half2* hv = reinterpret_cast<const __half2*>(&u);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 f = __half22float2(hv[e]);
+            ss += f.x * f.x + f.y * f.y;
           }
-          ss = warp_sum(ss);
-          const float rstd = rsqrtf(ss / static_cast<float>(p.K) + 1e-6f);
-          for (int c = lane * 4; c < kl; c += 128) {
-            const float4 v = *reinterpret_cast<const float4*>(xr + k0 + c);
-            const float4 g = *reinterpret_cast<const float4*>(p.gamma + k0 + c);
-            uint2 packed;
-            packed.x = pack_half2(v.x * rstd * g.x, v.y * rstd * g.y);
-            packed.y = pack_half2(v.z * rstd * g.z, v.w * rstd * g.w);
-            *reinterpret_cast<uint2*>(dst + c) = packed;
-          }
-        } else {
-          for (int c = lane * 4; c < kl; c += 128) *reinterpret_cast<uint2*>(dst + c) = make_uint2(0u, 0u);
         }
+        ss = warp_sum(ss);
+        if (lane == 0) s_rstd[r] = rsqrtf(ss / static_cast<float>(p.K) + 1e-6f);
       }
-    } else {
-      const int cpr = kl / 8;  // 16-byte chunks per row
-      for (int i = tid; i < kTokTile * cpr; i += kThreads) {
-        const int r = i / cpr;
-        const int c = (i - r * cpr) * 8;
-        const int m = m0 + r;
-        __half* dst = sA + static_cast<size_t>(r) * lda_s + c;
-        if (m < p.M) {
-          cp_async_16(smem_addr(dst), p.a + static_cast<size_t>(m) * p.lda + k0 + c);
-        } else {
-          *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
-        }
-      }
-      cp_async_commit();
-      cp_async_wait<0>();
     }
     __syncthreads();
 
@@ -157,6 +166,7 @@ __global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
       }
     }
 
+    __syncthreads();  // the activation tile becomes the reduction buffer
     // ---------------- cross-warp reduction through shared memory
 #pragma unroll
     for (int j = 0; j < NB; ++j) {
@@ -174,7 +184,8 @@ __global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
 
     auto red = [&](int n, int m) -> float {
       const float* r = sR + static_cast<size_t>(n) * kRedStride + m;
-      return r[0] + r[NT * kRedStride] + r[2 * NT * kRedStride] + r[3 * NT * kRedStride];
+      const float v = r[0] + r[NT * kRedStride] + r[2 * NT * kRedStride] + r[3 * NT * kRedStride];
+      return PRO == kProNorm ? v * s_rstd[m] : v;
     };
 
     // ---------------- epilogue
@@ -189,33 +200,37 @@ __global__ void __launch_bounds__(kThreads) gemm_ws_kernel(const GemmArgs p) {
         }
       }
     } else if (EPI == kEpiResidual) {
-      // this CTA's split partial -> warp-0 slice of sR, then cluster-wide ordered sum
-      for (int i = tid; i < NT * kTokTile; i += kThreads) {
-        const int n = i / kTokTile;
-        const int m = i - n * kTokTile;
-        sR[static_cast<size_t>(n) * kRedStride + m] = red(n, m);
-      }
+      // Split-K sum over the cluster, in split order: every CTA pushes the rows
+      // another rank owns into that rank's receive buffer (remote shared-memory
+      // stores), one cluster barrier, then each owner adds its rows locally.
       cg::cluster_group cluster = cg::this_cluster();
-      cluster.sync();
       const int n_split = static_cast<int>(cluster.num_blocks());
       const int rank = static_cast<int>(cluster.block_rank());
       const int rows_per = (kTokTile + n_split - 1) / n_split;
+      for (int i = tid; i < kTokTile * NT; i += kThreads) {
+        const int m = i / NT;
+        const int n = i - m * NT;
+        const int owner = m / rows_per;
+        float* dst = cluster.map_shared_rank(recv, owner);
+        dst[(static_cast<size_t>(rank) * rows_per + (m - owner * rows_per)) * NT + n] = red(n, m);
+      }
+      cluster.sync();
       const int r0 = rank * rows_per;
       const int r1 = min(kTokTile, r0 + rows_per);
       for (int i = tid; i < (r1 - r0) * NT; i += kThreads) {
-        const int m = r0 + i / NT;
-        const int n = i % NT;
+        const int mm = i / NT;
+        const int n = i - mm * NT;
+        const int m = r0 + mm;
         if (m0 + m < p.M) {
           float acc_s = 0.f;
-          for (int s = 0; s < n_split; ++s) {
-            const float* remote = cluster.map_shared_rank(sR, s);
-            acc_s += remote[static_cast<size_t>(n) * kRedStride + m];
-          }
-          float* xo = p.xo + static_cast<size_t>(m0 + m) * p.ldxo + nb0 * 16 + n;
-          *xo = *xo + acc_s;
+          for (int sp = 0; sp < n_split; ++sp) acc_s += recv[(static_cast<size_t>(sp) * rows_per + mm) * NT + n];
+          const size_t idx = static_cast<size_t>(m0 + m) * p.ldxo + nb0 * 16 + n;
+          const float xn = p.xo[idx] + acc_s;
+          p.xo[idx] = xn;
+          p.xo16[idx] = __float2half_rn(xn);
         }
       }
-      cluster.sync();  // remote reads done before any CTA reuses or releases its shared memory
+      cluster.sync();  // receive buffers are refilled by the next m-tile only after every owner summed
     } else {  // kEpiSwiglu: block j rows 0..7 = gate of h columns (nb0+j)*8 + r, rows 8..15 = up
       constexpr int NH = NB * 8;
       for (int i = tid; i < NH * kTokTile; i += kThreads) {
@@ -245,6 +260,7 @@ const void* select_kernel(int nb, int pro, int epi) {
   if (nb == NB_ && pro == PRO_ && epi == EPI_) return kernel_ptr<NB_, PRO_, EPI_>();
   FSX_SEL(1, kProNorm, kEpiStore)
   FSX_SEL(2, kProNorm, kEpiStore)
+  FSX_SEL(3, kProNorm, kEpiStore)
   FSX_SEL(1, kProNorm, kEpiSwiglu)
   FSX_SEL(2, kProNorm, kEpiSwiglu)
   FSX_SEL(1, kProCopy, kEpiResidual)
@@ -258,7 +274,7 @@ const void* select_kernel(int nb, int pro, int epi) {
 }  // namespace
 
 cudaError_t gemm_set_attributes() {
-  const int nbs[2] = {1, 2};
+  const int nbs[3] = {1, 2, 3};
   const int pros[2] = {kProNorm, kProCopy};
   const int epis[3] = {kEpiStore, kEpiResidual, kEpiSwiglu};
   for (int nb : nbs)
@@ -292,7 +308,7 @@ GemmPlan plan_gemm(int n_rows, int K, int M, int nb, int ks, int prologue, int e
   const int per = (m_tiles + nz - 1) / nz;
   nz = (m_tiles + per - 1) / per;
   pl.grid = dim3(nx, ny, nz);
-  pl.smem = gemm_smem_bytes(nb, ks);
+  pl.smem = gemm_smem_bytes(nb, pl.ks, epilogue);
   return pl;
 }
 
@@ -309,7 +325,7 @@ cudaError_t launch_gemm(const GemmPlan& pl, const GemmArgs& args_in, cudaStream_
 }
 
 cudaError_t launch_ex(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool pdl,
-                      void** args, int cluster_y) {
+                      void** args, int cluster_y, int cluster_x) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
@@ -322,9 +338,9 @@ cudaError_t launch_ex(const void* fn, dim3 grid, dim3 block, size_t smem, cudaSt
     attr[n].val.programmaticStreamSerializationAllowed = 1;
     ++n;
   }
-  if (cluster_y > 1) {
+  if (cluster_y > 1 || cluster_x > 1) {
     attr[n].id = cudaLaunchAttributeClusterDimension;
-    attr[n].val.clusterDim.x = 1;
+    attr[n].val.clusterDim.x = static_cast<unsigned>(cluster_x);
     attr[n].val.clusterDim.y = static_cast<unsigned>(cluster_y);
     attr[n].val.clusterDim.z = 1;
     ++n;

@@ -35,18 +35,20 @@ struct GemmArgs {
   int ks;              // K per split (multiple of 64); the last split may be shorter
   int M;               // activation rows
   int m_tiles_per_cta; // 48-row tiles per CTA along grid.z
-  // prologue kProNorm: A = RMSNorm(x) * gamma computed from fp32 rows of length K
-  const float* x;
-  const float* gamma;
-  int ldx;
+  // prologue kProNorm: A = fp16 copy of the residual stream (rows of length K);
+  // the norm gain is folded into w and the epilogue scales by the row's 1/rms
+  const __half* x16;
+  int ldx16;
   // prologue kProCopy: A = fp16 rows
   const __half* a;
   int lda;
   // epilogue kEpiStore: y[m, n] fp16; kEpiSwiglu: y[m, n/2] = silu(gate) * up fp16
   __half* y;
   int ldy;
-  // epilogue kEpiResidual: xo[m, n] += sum over the K splits (one cluster), fp32
+  // epilogue kEpiResidual: xo[m, n] += sum over the K splits (one cluster), fp32,
+  // and xo16[m, n] = fp16 copy of the updated value
   float* xo;
+  __half* xo16;
   int ldxo;
   int* status;
 };
@@ -104,6 +106,7 @@ struct EmbedArgs {
   int B;
   long long max_total;
   float* x;               // [B*T, d]
+  __half* x16;            // fp16 copy of x
   int* status;
 };
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t stream, bool pdl);
@@ -121,8 +124,8 @@ struct HeadArgs {
 cudaError_t launch_head(const HeadArgs& a, cudaStream_t stream, bool pdl);
 
 // Launch helper: cudaLaunchKernelEx with the programmatic-stream-serialisation
-// attribute when `pdl` is set and a (1, cluster_y, 1) cluster when cluster_y > 1.
+// attribute when `pdl` is set and a (cluster_x, cluster_y, 1) cluster when either exceeds 1.
 cudaError_t launch_ex(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
-                      bool pdl, void** args, int cluster_y = 1);
+                      bool pdl, void** args, int cluster_y = 1, int cluster_x = 1);
 
 }  // namespace fsx

@@ -27,7 +27,7 @@ FSX_ERR_DEVICE_ARG = 6
 FSX_F32 = 0
 FSX_BF16 = 1
 
-KCLASS = {"qkv": 0, "attention": 1, "out_proj": 2, "gate_up": 3, "down": 4}
+KCLASS = {"qkv": 0, "attention": 1, "out_proj": 2, "gate_up": 3, "down": 4, "persistent": 5}
 
 
 class FsxError(RuntimeError):

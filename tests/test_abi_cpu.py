@@ -115,12 +115,13 @@ def test_tick_rejects_null_handle(lib):
 
 
 def test_attention_host_validation(lib):
-    ws = fsx.attention_workspace_bytes(2, 32, 42, 4)
-    assert ws == 256 + 2 * 32 * 4 * 48 * 128 * 4 + 2 * 32 * 4 * 48 * 4
+    ws = fsx.attention_workspace_bytes(2, 32, 42, 12)
+    assert ws == 256 + 2 * 32 * 12 * 48 * 128 * 4 + 2 * 32 * 12 * 48 * 4
     assert fsx.attention_workspace_bytes(2, 32, 42, 1) == 256
+    assert fsx.attention_workspace_bytes(2, 32, 42, 8) == 256  # up to 8 splits merge on chip
     fake = 1 << 20  # never dereferenced: every case fails host validation first
     base = dict(q=fake, qs=4096 * 3, ko=fake, vo=fake, os=4096 * 3, nq=42, no=42, kc=fake, vc=fake, dt=1,
-                off=fake, B=2, H=32, D=128, S=4, out=fake, lse=None, ws=fake, wsb=ws)
+                off=fake, B=2, H=32, D=128, S=12, out=fake, lse=None, ws=fake, wsb=ws)
 
     def call(**kw):
         a = dict(base, **kw)

@@ -20,14 +20,20 @@ SMALL = synth.Dims(n_layers=4)
 def _parity(case, vehicles=None, max_batch=None):
     ex = case.expert(max_batch)
     try:
+        launches = ex.launches(case.B)
         wp, att = fc.run_debug_tick(ex, case)
         wp_graph = fc.run_tick(ex, case)
     finally:
         ex.close()
     assert np.isfinite(wp).all()
-    # graph replay and the kernel-by-kernel debug path run the same kernels in
-    # the same order with deterministic reductions: bit-identical waypoints
-    assert np.array_equal(wp_graph, wp)
+    if launches > 1:
+        # multi-kernel path: graph replay and the kernel-by-kernel debug path run
+        # the same kernels in the same order with deterministic reductions
+        assert np.array_equal(wp_graph, wp)
+    else:
+        # single-launch persistent path: residual updates are fp32 atomics, so
+        # two ticks agree to rounding (amplified by the 32-layer stack)
+        assert np.linalg.norm(wp_graph - wp) <= 5e-3 * np.linalg.norm(wp)
     worst = []
     for b in (range(case.B) if vehicles is None else vehicles):
         worst.append(fc.check_vehicle(case, b, wp, att))
