@@ -17,7 +17,7 @@
  *   - Every function returns an fsx_status; on failure a thread-local message
  *     is available from fsx_last_error(). Host-side argument checks happen
  *     before anything is enqueued.
- *   - Supported shapes: head_dim == 128, d_model % 64 == 0, d_model <= 1024,
+ *   - Supported shapes: head_dim == 128, d_model % 128 == 0, d_model <= 1024,
  *     d_ff % 64 == 0, 1 <= n_action + n_frame <= 48, 1 <= n_waypoints <=
  *     n_action + n_frame, n_layers <= 128. Other shapes give FSX_ERR_UNSUPPORTED.
  *   - Precision: weights are stored as fp16 (round-to-nearest-even from the

@@ -28,6 +28,7 @@ __global__ void embed_kernel(const EmbedArgs a) {
   }
   float* xr = a.x + static_cast<size_t>(row) * a.d;
   const float* pos = a.pos_emb + static_cast<size_t>(t) * a.d;
+  __shared__ float s_part[4];
   for (int c = threadIdx.x; c < a.d; c += blockDim.x) {
     float v;
     if (t < a.n_action) {
@@ -43,6 +44,13 @@ __global__ void embed_kernel(const EmbedArgs a) {
     const float xv = v + pos[c];
     xr[c] = xv;
     a.x16[static_cast<size_t>(row) * a.d + c] = __float2half_rn(xv);
+    // sum of x^2 over this 128-column group (blockDim.x == 128: one group per pass)
+    const float ws = warp_sum(xv * xv);
+    if ((threadIdx.x & 31) == 0) s_part[threadIdx.x >> 5] = ws;
+    __syncthreads();
+    if (threadIdx.x == 0)
+      a.ss[static_cast<size_t>(c / 128) * a.ss_stride + row] = s_part[0] + s_part[1] + s_part[2] + s_part[3];
+    __syncthreads();
   }
 }
 

@@ -22,6 +22,7 @@
 #include <vector>
 
 #include "../../include/fsx.h"
+#include "gemm_tc.h"
 #include "kernels.h"
 #include "persistent.h"
 
@@ -64,7 +65,9 @@ struct fsx_handle_s {
   // packed fp16 weights
   void* w_arena = nullptr;
   long long weight_bytes = 0;
-  std::vector<const uint4*> w_qkv, w_o, w_gu, w_dn;
+  std::vector<const unsigned char*> w_qkv, w_o, w_gu, w_dn;  // tcgen05 tile images per layer
+  // 2-D tensor maps of the activation buffers for the token tile sizes 48 / 128 / 256
+  CUtensorMap map_x16[3], map_o[3], map_h[3];
   // fp32 small parameters
   float* params = nullptr;
   float *act_emb = nullptr, *pos_emb = nullptr, *attn_norm = nullptr, *mlp_norm = nullptr;
@@ -72,6 +75,8 @@ struct fsx_handle_s {
   // workspace
   float* x = nullptr;
   __half* x16 = nullptr;
+  float* ss = nullptr;   // per-row sums of x^2 over 128-column groups
+  int ss_stride = 0;
   __half* qkv = nullptr;
   __half* o = nullptr;
   __half* hbuf = nullptr;
@@ -126,7 +131,7 @@ fsx_status check_config(const fsx_config* c) {
   const int T = c->n_action + c->n_frame;
   if (c->n_waypoints > T) return fail(FSX_ERR_INVALID_ARG, "n_waypoints exceeds the token count");
   if (c->head_dim != fsx::kHeadDim) return fail(FSX_ERR_UNSUPPORTED, "head_dim must be 128");
-  if (c->d_model % 64 != 0 || c->d_model > 1024) return fail(FSX_ERR_UNSUPPORTED, "d_model must be a multiple of 64, <= 1024");
+  if (c->d_model % 128 != 0 || c->d_model > 1024) return fail(FSX_ERR_UNSUPPORTED, "d_model must be a multiple of 128, <= 1024");
   if (c->d_ff % 64 != 0) return fail(FSX_ERR_UNSUPPORTED, "d_ff must be a multiple of 64");
   if (T > fsx::kTokTile) return fail(FSX_ERR_UNSUPPORTED, "n_action + n_frame must be <= 48");
   if (c->n_layers > fsx::kMaxLayers) return fail(FSX_ERR_UNSUPPORTED, "n_layers must be <= 128");
@@ -230,30 +235,32 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
   ea.max_total = c.max_total_cache_tokens;
   ea.x = h->x;
   ea.x16 = h->x16;
+  ea.ss = h->ss;
+  ea.ss_stride = h->ss_stride;
   ea.status = h->status;
   FSX_CUDA(fsx::launch_embed(ea, st, pdl));
 
   // 48-row QKV tiles: 256 CTAs at two per SM run as one wave
-  const fsx::GemmPlan pq = fsx::plan_gemm(3 * HD, d, M, 3, d, fsx::kProNorm, fsx::kEpiStore, h->sm_count);
-  const fsx::GemmPlan po = fsx::plan_gemm(d, HD, M, 2, 512, fsx::kProCopy, fsx::kEpiResidual, h->sm_count);
-  const fsx::GemmPlan pg = fsx::plan_gemm(2 * F, d, M, 1, d, fsx::kProNorm, fsx::kEpiSwiglu, h->sm_count);
-  const fsx::GemmPlan pd = fsx::plan_gemm(d, F, M, 1, 256, fsx::kProCopy, fsx::kEpiResidual, h->sm_count);
+  // token tile of the tensor-core GEMMs: 48 for one vehicle, then 128 / 256
+  const int bn_i = M <= 48 ? 0 : (M <= 1024 ? 1 : 2);
+  const int bn = bn_i == 0 ? 48 : (bn_i == 1 ? 128 : 256);
   const int S = attention_splits(h, B);
 
   for (int l = 0; l < c.n_layers; ++l) {
-    fsx::GemmArgs g{};
+    fsx::TcGemmArgs g{};
     g.M = M;
     g.status = h->status;
-    // RMSNorm + [W_q; W_k; W_v]
+    // RMSNorm + [W_q; W_k; W_v] (norm gain folded into the tiles)
     g.w = h->w_qkv[l];
-    g.n_rows = 3 * HD;
+    g.N = 3 * HD;
     g.K = d;
-    g.x16 = h->x16;
-    g.ldx16 = d;
     g.y = h->qkv;
     g.ldy = 3 * HD;
+    g.ss_in = h->ss;
+    g.n_ss = d / 128;
+    g.ss_stride = h->ss_stride;
     FSX_CUDA(mark(kClassQkv, true));
-    FSX_CUDA(fsx::launch_gemm(pq, g, st, pdl));
+    FSX_CUDA(fsx::launch_gemm_tc(h->map_x16[bn_i], g, bn, fsx::kEpiStore, true, st, pdl));
     FSX_CUDA(mark(kClassQkv, false));
 
     // Eq. 1 over [cache_l ; own]
@@ -285,50 +292,51 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     }
 
     // x += o W_o^T
-    fsx::GemmArgs go{};
+    fsx::TcGemmArgs go{};
     go.M = M;
     go.status = h->status;
     go.w = h->w_o[l];
-    go.n_rows = d;
+    go.N = d;
     go.K = HD;
-    go.a = h->o;
-    go.lda = HD;
     go.xo = h->x;
     go.xo16 = h->x16;
     go.ldxo = d;
+    go.ss_out = h->ss;
+    go.ss_stride = h->ss_stride;
     FSX_CUDA(mark(kClassWo, true));
-    FSX_CUDA(fsx::launch_gemm(po, go, st, pdl));
+    FSX_CUDA(fsx::launch_gemm_tc(h->map_o[bn_i], go, bn, fsx::kEpiResidual, false, st, pdl));
     FSX_CUDA(mark(kClassWo, false));
 
     // h = silu(RMSNorm(x) W_g^T) * (RMSNorm(x) W_u^T)
-    fsx::GemmArgs gg{};
+    fsx::TcGemmArgs gg{};
     gg.M = M;
     gg.status = h->status;
     gg.w = h->w_gu[l];
-    gg.n_rows = 2 * F;
+    gg.N = 2 * F;
     gg.K = d;
-    gg.x16 = h->x16;
-    gg.ldx16 = d;
     gg.y = h->hbuf;
     gg.ldy = F;
+    gg.ss_in = h->ss;
+    gg.n_ss = d / 128;
+    gg.ss_stride = h->ss_stride;
     FSX_CUDA(mark(kClassGateUp, true));
-    FSX_CUDA(fsx::launch_gemm(pg, gg, st, pdl));
+    FSX_CUDA(fsx::launch_gemm_tc(h->map_x16[bn_i], gg, bn, fsx::kEpiSwiglu, true, st, pdl));
     FSX_CUDA(mark(kClassGateUp, false));
 
     // x += h W_d^T
-    fsx::GemmArgs gd{};
+    fsx::TcGemmArgs gd{};
     gd.M = M;
     gd.status = h->status;
     gd.w = h->w_dn[l];
-    gd.n_rows = d;
+    gd.N = d;
     gd.K = F;
-    gd.a = h->hbuf;
-    gd.lda = F;
     gd.xo = h->x;
     gd.xo16 = h->x16;
     gd.ldxo = d;
+    gd.ss_out = h->ss;
+    gd.ss_stride = h->ss_stride;
     FSX_CUDA(mark(kClassDown, true));
-    FSX_CUDA(fsx::launch_gemm(pd, gd, st, pdl));
+    FSX_CUDA(fsx::launch_gemm_tc(h->map_h[bn_i], gd, bn, fsx::kEpiResidual, false, st, pdl));
     FSX_CUDA(mark(kClassDown, false));
   }
 
@@ -423,7 +431,7 @@ void free_handle(fsx_handle_s* h) {
   for (cudaEvent_t e : h->tev) cudaEventDestroy(e);
   if (h->last_tick) cudaEventDestroy(h->last_tick);
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
-  void* bufs[] = {h->p_arena, h->p_x, h->p_counters, h->w_arena, h->params, h->x, h->x16, h->qkv, h->o, h->hbuf, h->part, h->status, h->d_args,
+  void* bufs[] = {h->p_arena, h->p_x, h->p_counters, h->w_arena, h->params, h->x, h->x16, h->ss, h->qkv, h->o, h->hbuf, h->part, h->status, h->d_args,
                   h->st_offsets, h->st_frames, h->st_waypoints};
   for (void* p : bufs)
     if (p) cudaFree(p);
@@ -474,48 +482,58 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
 
   FSX_CUDA_H(cudaSetDevice(device));
   FSX_CUDA_H(cudaDeviceGetAttribute(&h->sm_count, cudaDevAttrMultiProcessorCount, device));
-  FSX_CUDA_H(fsx::gemm_set_attributes());
+  FSX_CUDA_H(fsx::gemm_tc_set_attributes());
   FSX_CUDA_H(fsx::attention_set_attributes());
 
-  // ---- packed fp16 weights: per layer [qkv | o | gate/up | down], 256-byte aligned
-  const size_t n_qkv = static_cast<size_t>(3) * HD * d, n_o = static_cast<size_t>(d) * HD;
-  const size_t n_gu = static_cast<size_t>(2) * F * d, n_dn = static_cast<size_t>(d) * F;
-  const size_t b_qkv = align_up(n_qkv * 2, 256), b_o = align_up(n_o * 2, 256);
-  const size_t b_gu = align_up(n_gu * 2, 256), b_dn = align_up(n_dn * 2, 256);
-  const size_t per_layer = b_qkv + b_o + b_gu + b_dn;
+  // ---- tcgen05 weight tiles: per layer [QKV | W_o | gate/up | W_d], each matrix as
+  // 128-row x 64-K tiles in the swizzled shared-memory image (n-tile major)
+  const size_t tile = fsx::kTcTileBytes;
+  const size_t t_qkv = static_cast<size_t>(3 * HD / 128) * (d / 64), t_o = static_cast<size_t>(d / 128) * (HD / 64);
+  const size_t t_gu = static_cast<size_t>(2 * F / 128) * (d / 64), t_dn = static_cast<size_t>(d / 128) * (F / 64);
+  const size_t per_layer = (t_qkv + t_o + t_gu + t_dn) * tile;
   const size_t arena = per_layer * L;
-  h->weight_bytes = static_cast<long long>((n_qkv + n_o + n_gu + n_dn) * 2 * L);
+  h->weight_bytes = static_cast<long long>(arena);
   FSX_CUDA_H(cudaMalloc(&h->w_arena, arena));
   {
     std::vector<__half> host(arena / 2);
     const size_t hd_d = static_cast<size_t>(HD) * d;
+    // rows(r) -> source row r of the (row-permuted) matrix; K columns; optional per-K gain
+    auto pack_matrix = [&](auto rows, int N, int K, const float* gain, unsigned char* out) {
+      const float* rp[128];
+      for (int nt = 0; nt < N / 128; ++nt)
+        for (int kt = 0; kt < K / 64; ++kt) {
+          for (int r = 0; r < 128; ++r) rp[r] = rows(nt * 128 + r);
+          fsx::pack_tc_tile(rp, gain, kt * 64,
+                            reinterpret_cast<__half*>(out + (static_cast<size_t>(nt) * (K / 64) + kt) * tile));
+        }
+    };
     auto pack_layer = [&](int l) {
       unsigned char* base = reinterpret_cast<unsigned char*>(host.data()) + per_layer * l;
       const float* wq = w->wq + hd_d * l;
       const float* wk = w->wk + hd_d * l;
       const float* wv = w->wv + hd_d * l;
-      pack_fragments(
+      pack_matrix(
           [&](int r) -> const float* {
             if (r < HD) return wq + static_cast<size_t>(r) * d;
             if (r < 2 * HD) return wk + static_cast<size_t>(r - HD) * d;
             return wv + static_cast<size_t>(r - 2 * HD) * d;
           },
-          3 * HD, d, reinterpret_cast<__half*>(base), w->attn_norm + static_cast<size_t>(l) * d);
+          3 * HD, d, w->attn_norm + static_cast<size_t>(l) * d, base);
       const float* wo = w->wo + hd_d * l;
-      pack_fragments([&](int r) -> const float* { return wo + static_cast<size_t>(r) * HD; }, d, HD,
-                     reinterpret_cast<__half*>(base + b_qkv));
+      pack_matrix([&](int r) -> const float* { return wo + static_cast<size_t>(r) * HD; }, d, HD, nullptr,
+                  base + t_qkv * tile);
       const float* wg = w->w_gate + static_cast<size_t>(F) * d * l;
       const float* wu = w->w_up + static_cast<size_t>(F) * d * l;
       // packed row p: block p/16, rows 0..7 gate rows 8*(p/16)+r, rows 8..15 the matching up rows
-      pack_fragments(
-          [&](int p) -> const float* {
-            const int blk = p >> 4, r = p & 15;
+      pack_matrix(
+          [&](int q) -> const float* {
+            const int blk = q >> 4, r = q & 15;
             return r < 8 ? wg + static_cast<size_t>(blk * 8 + r) * d : wu + static_cast<size_t>(blk * 8 + r - 8) * d;
           },
-          2 * F, d, reinterpret_cast<__half*>(base + b_qkv + b_o), w->mlp_norm + static_cast<size_t>(l) * d);
+          2 * F, d, w->mlp_norm + static_cast<size_t>(l) * d, base + (t_qkv + t_o) * tile);
       const float* wd = w->w_down + static_cast<size_t>(d) * F * l;
-      pack_fragments([&](int r) -> const float* { return wd + static_cast<size_t>(r) * F; }, d, F,
-                     reinterpret_cast<__half*>(base + b_qkv + b_o + b_gu));
+      pack_matrix([&](int r) -> const float* { return wd + static_cast<size_t>(r) * F; }, d, F, nullptr,
+                  base + (t_qkv + t_o + t_gu) * tile);
     };
     const int n_threads = std::max(1, std::min<int>(16, static_cast<int>(std::thread::hardware_concurrency())));
     std::vector<std::thread> pool;
@@ -528,10 +546,10 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
   }
   for (int l = 0; l < L; ++l) {
     const unsigned char* base = static_cast<const unsigned char*>(h->w_arena) + per_layer * l;
-    h->w_qkv.push_back(reinterpret_cast<const uint4*>(base));
-    h->w_o.push_back(reinterpret_cast<const uint4*>(base + b_qkv));
-    h->w_gu.push_back(reinterpret_cast<const uint4*>(base + b_qkv + b_o));
-    h->w_dn.push_back(reinterpret_cast<const uint4*>(base + b_qkv + b_o + b_gu));
+    h->w_qkv.push_back(base);
+    h->w_o.push_back(base + t_qkv * tile);
+    h->w_gu.push_back(base + (t_qkv + t_o) * tile);
+    h->w_dn.push_back(base + (t_qkv + t_o + t_gu) * tile);
   }
 
   // ---- stream-ordered weights of the persistent single-vehicle tick
@@ -635,12 +653,27 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
 
   // ---- workspace for max_batch
   const size_t Mmax = static_cast<size_t>(cfg->max_batch) * T;
-  const size_t m_pad = (Mmax + fsx::kTokTile - 1) / fsx::kTokTile * fsx::kTokTile;
+  const size_t m_pad = (Mmax + 255) / 256 * 256;  // whole token tiles of every GEMM tile size
   FSX_CUDA_H(cudaMalloc(&h->x, m_pad * d * sizeof(float)));
   FSX_CUDA_H(cudaMalloc(&h->x16, m_pad * d * sizeof(__half)));
+  h->ss_stride = static_cast<int>(m_pad);
+  FSX_CUDA_H(cudaMalloc(&h->ss, static_cast<size_t>(d / 128) * m_pad * sizeof(float)));
+  FSX_CUDA_H(cudaMemset(h->ss, 0, static_cast<size_t>(d / 128) * m_pad * sizeof(float)));
   FSX_CUDA_H(cudaMalloc(&h->qkv, m_pad * 3 * HD * sizeof(__half)));
   FSX_CUDA_H(cudaMalloc(&h->o, m_pad * HD * sizeof(__half)));
   FSX_CUDA_H(cudaMalloc(&h->hbuf, m_pad * F * sizeof(__half)));
+  FSX_CUDA_H(cudaMemset(h->x16, 0, m_pad * d * sizeof(__half)));
+  FSX_CUDA_H(cudaMemset(h->o, 0, m_pad * HD * sizeof(__half)));
+  FSX_CUDA_H(cudaMemset(h->hbuf, 0, m_pad * F * sizeof(__half)));
+  {
+    const uint32_t boxes[3] = {48, 128, 256};
+    for (int i = 0; i < 3; ++i) {
+      if (!fsx::encode_act_map(&h->map_x16[i], h->x16, m_pad, d, boxes[i]) ||
+          !fsx::encode_act_map(&h->map_o[i], h->o, m_pad, HD, boxes[i]) ||
+          !fsx::encode_act_map(&h->map_h[i], h->hbuf, m_pad, F, boxes[i]))
+        return bail(fail(FSX_ERR_CUDA, "tensor map encoding of the activation buffers failed"));
+    }
+  }
   size_t part = 0;
   for (int B = 1; B <= cfg->max_batch; ++B)
     part = std::max(part, fsx::attention_workspace_bytes(B, cfg->n_heads, attention_splits(h, B)));

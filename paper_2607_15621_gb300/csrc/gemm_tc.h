@@ -1,0 +1,44 @@
+// Launch interface of the tcgen05 projection GEMMs (gemm_tc.cu).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "kernels.h"
+
+namespace fsx {
+
+constexpr int kTcTileRows = 128;  // weight rows per tile
+constexpr int kTcTileK = 64;      // K per tile
+constexpr int kTcTileBytes = kTcTileRows * kTcTileK * 2;
+
+struct TcGemmArgs {
+  const unsigned char* w;  // packed tiles: tile (n_tile, k_tile) at (n_tile * K/64 + k_tile) * 16 KB
+  int N;                   // weight rows (multiple of 128)
+  int K;                   // reduction length (multiple of 64)
+  int M;                   // tokens
+  __half* y;               // kEpiStore: y[m, n]; kEpiSwiglu: y[m, n / 2]
+  int ldy;
+  float* xo;               // kEpiResidual: xo[m, n] += result, xo16 = fp16 copy
+  __half* xo16;
+  int ldxo;
+  // sums of x^2 per token over 128-column groups: [n_ss][ss_stride], group j = columns 128j..128j+127.
+  // kEpiResidual writes group blockIdx.x of the updated rows; RMSNorm-fused GEMMs read all groups.
+  float* ss_out;
+  const float* ss_in;
+  int n_ss;
+  int ss_stride;
+  int* status;
+};
+
+cudaError_t gemm_tc_set_attributes();
+cudaError_t launch_gemm_tc(const CUtensorMap& map_a, const TcGemmArgs& args, int bn, int epi, bool norm,
+                           cudaStream_t stream, bool pdl);
+// rows[128]: pointers to the 128 source rows (fp32, length >= k0 + 64); col_scale: optional per-K gain.
+void pack_tc_tile(const float* const* rows, const float* col_scale, int k0, __half* out);
+// 2-D fp16 tensor map over a row-major [rows, cols] buffer with a (box_rows x 64) box and 128-byte swizzle.
+bool encode_act_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
+
+}  // namespace fsx

@@ -23,48 +23,9 @@ struct TickArgs {
   float* waypoints;
 };
 
-// ------------------------------------------------------------------ GEMM
-// Y[M, N] = A[M, K] . W[N, K]^T with W packed as 16x16 fp16 fragment blocks.
-enum GemmPrologue { kProNorm = 0, kProCopy = 1 };
+// ------------------------------------------------------------ epilogues
+// Epilogues of the tensor-core projection GEMMs (gemm_tc.cu).
 enum GemmEpilogue { kEpiStore = 0, kEpiResidual = 1, kEpiSwiglu = 2 };
-
-struct GemmArgs {
-  const uint4* w;      // packed weights: block (nb, kb) = 32 x uint4 at (nb * K/16 + kb) * 32
-  int n_rows;          // packed rows N (multiple of 16)
-  int K;               // reduction length (multiple of 64)
-  int ks;              // K per split (multiple of 64); the last split may be shorter
-  int M;               // activation rows
-  int m_tiles_per_cta; // 48-row tiles per CTA along grid.z
-  // prologue kProNorm: A = fp16 copy of the residual stream (rows of length K);
-  // the norm gain is folded into w and the epilogue scales by the row's 1/rms
-  const __half* x16;
-  int ldx16;
-  // prologue kProCopy: A = fp16 rows
-  const __half* a;
-  int lda;
-  // epilogue kEpiStore: y[m, n] fp16; kEpiSwiglu: y[m, n/2] = silu(gate) * up fp16
-  __half* y;
-  int ldy;
-  // epilogue kEpiResidual: xo[m, n] += sum over the K splits (one cluster), fp32,
-  // and xo16[m, n] = fp16 copy of the updated value
-  float* xo;
-  __half* xo16;
-  int ldxo;
-  int* status;
-};
-
-struct GemmPlan {
-  int nb;       // 16-row blocks per CTA (1 or 2)
-  int ks;
-  int prologue;
-  int epilogue;
-  dim3 grid;
-  size_t smem;
-};
-
-GemmPlan plan_gemm(int n_rows, int K, int M, int nb, int ks, int prologue, int epilogue, int sm_count);
-cudaError_t launch_gemm(const GemmPlan& plan, const GemmArgs& args, cudaStream_t stream, bool pdl);
-cudaError_t gemm_set_attributes();
 
 // ------------------------------------------------------------- attention
 struct AttnArgs {
@@ -107,6 +68,8 @@ struct EmbedArgs {
   long long max_total;
   float* x;               // [B*T, d]
   __half* x16;            // fp16 copy of x
+  float* ss;              // per-row sums of x^2 over 128-column groups, [d/128][ss_stride]
+  int ss_stride;
   int* status;
 };
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t stream, bool pdl);

@@ -87,12 +87,42 @@ __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
-// Device-wide arrival counter: every thread's prior global writes are fenced,
-// then one thread adds 1.
+// Device-wide arrival counter: after the CTA barrier one thread adds 1 with
+// release semantics, which publishes the CTA's earlier global writes.
 __device__ __forceinline__ void arrive(int* counter) {
-  __threadfence();
   __syncthreads();
-  if (threadIdx.x == 0) atomicAdd(counter, 1);
+  if (threadIdx.x == 0) asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(counter) : "memory");
+}
+
+// Address of the same shared-memory offset in cluster CTA `rank`.
+__device__ __forceinline__ uint32_t cluster_addr(const void* local, int rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(local)), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void st_cluster_v4(uint32_t addr, uint4 v) {
+  asm volatile("st.shared::cluster.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+
+// Copy rows x bytes_per_row (multiple of 16) starting at the same local offset to
+// the 3 partner CTAs of the cluster (16-byte remote stores).
+__device__ __forceinline__ void push_rows(const void* base, int rows, int row_stride_bytes, int bytes_per_row,
+                                          int my_rank, int tid, int nthr) {
+  const int upr = bytes_per_row / 16;
+  const unsigned char* b = static_cast<const unsigned char*>(base);
+  for (int i = tid; i < rows * upr * (kPersistCluster - 1); i += nthr) {
+    const int peer_i = i / (rows * upr);
+    const int rest = i - peer_i * rows * upr;
+    const int r = rest / upr;
+    const int u = rest - r * upr;
+    const int peer = peer_i + (peer_i >= my_rank ? 1 : 0);
+    const unsigned char* src = b + static_cast<size_t>(r) * row_stride_bytes + u * 16;
+    st_cluster_v4(cluster_addr(src, peer), *reinterpret_cast<const uint4*>(src));
+  }
 }
 
 // Bounded wait until *counter >= target (one thread polls, the CTA follows).
@@ -239,7 +269,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   }
   arrive(p.counters + 0);
 
-  // x (state buffer) -> RMSNorm -> fp16 rows in every partner's activation tile
+  // x (state buffer) -> RMSNorm -> fp16 rows in every partner's activation tile:
+  // this rank normalises rows 12r..12r+11 into its own tile and copies them out
   auto load_normalized = [&](const float* Xs) {
     const int r0 = rank * kRowsPerRank;
     const int r1 = min(r0 + kRowsPerRank, T);
@@ -248,25 +279,28 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       float4 v[8];
       float ss = 0.f;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int c = lane * 4 + j * 128;
+      for (int j = 0; j < 4; ++j) {  // lane holds 8 consecutive values per 256-wide slab
+        const int c = lane * 8 + j * 256;
         if (c < d) {
-          v[j] = ld_cg4(xr + c);
-          ss += v[j].x * v[j].x + v[j].y * v[j].y + v[j].z * v[j].z + v[j].w * v[j].w;
+          v[2 * j] = ld_cg4(xr + c);
+          v[2 * j + 1] = ld_cg4(xr + c + 4);
+          ss += v[2 * j].x * v[2 * j].x + v[2 * j].y * v[2 * j].y + v[2 * j].z * v[2 * j].z + v[2 * j].w * v[2 * j].w;
+          ss += v[2 * j + 1].x * v[2 * j + 1].x + v[2 * j + 1].y * v[2 * j + 1].y + v[2 * j + 1].z * v[2 * j + 1].z +
+                v[2 * j + 1].w * v[2 * j + 1].w;
         }
       }
       ss = warp_sum(ss);
       const float rstd = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int c = lane * 4 + j * 128;
+      for (int j = 0; j < 4; ++j) {
+        const int c = lane * 8 + j * 256;
         if (c < d) {
-          uint2 pk;
-          pk.x = pack_half2(v[j].x * rstd, v[j].y * rstd);
-          pk.y = pack_half2(v[j].z * rstd, v[j].w * rstd);
-#pragma unroll
-          for (int dst = 0; dst < kCl; ++dst)
-            *reinterpret_cast<uint2*>(cluster.map_shared_rank(act, dst) + static_cast<size_t>(r) * as + c) = pk;
+          uint4 pk;
+          pk.x = pack_half2(v[2 * j].x * rstd, v[2 * j].y * rstd);
+          pk.y = pack_half2(v[2 * j].z * rstd, v[2 * j].w * rstd);
+          pk.z = pack_half2(v[2 * j + 1].x * rstd, v[2 * j + 1].y * rstd);
+          pk.w = pack_half2(v[2 * j + 1].z * rstd, v[2 * j + 1].w * rstd);
+          *reinterpret_cast<uint4*>(act + static_cast<size_t>(r) * as + c) = pk;
         }
       }
     }
@@ -274,6 +308,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       const int r = T + i / (d / 8);
       *reinterpret_cast<uint4*>(act + static_cast<size_t>(r) * as + (i % (d / 8)) * 8) = make_uint4(0u, 0u, 0u, 0u);
     }
+    __syncthreads();
+    if (r1 > r0) push_rows(act + static_cast<size_t>(r0) * as, r1 - r0, as * 2, d * 2, rank, tid, kThr);
     cluster.sync();
   };
 
@@ -347,24 +383,24 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       block_gemm(w, d / 16, act, as, acc, lane);
       const int kind = warp >> 1;                       // 0 q, 1 k, 2 v
       const int dim = rank * 32 + (warp & 1) * 16 + (lane >> 2);
-      __half* dstbuf = kind == 0 ? qbuf : (kind == 1 ? ownk : ownv);
+      __half* b = kind == 0 ? qbuf : (kind == 1 ? ownk : ownv);
 #pragma unroll
       for (int t = 0; t < 6; ++t) {
         const int m = t * 8 + 2 * (lane & 3);
-#pragma unroll
-        for (int dst = 0; dst < kCl; ++dst) {
-          __half* b = cluster.map_shared_rank(dstbuf, dst);
-          b[m * kQS + dim] = __float2half_rn(acc[t][0]);
-          b[(m + 1) * kQS + dim] = __float2half_rn(acc[t][1]);
-          b[m * kQS + dim + 8] = __float2half_rn(acc[t][2]);
-          b[(m + 1) * kQS + dim + 8] = __float2half_rn(acc[t][3]);
-        }
+        b[m * kQS + dim] = __float2half_rn(acc[t][0]);
+        b[(m + 1) * kQS + dim] = __float2half_rn(acc[t][1]);
+        b[m * kQS + dim + 8] = __float2half_rn(acc[t][2]);
+        b[(m + 1) * kQS + dim + 8] = __float2half_rn(acc[t][3]);
       }
     }
     __syncthreads();
     if (tid == 0)
       for (int i = 0; i < 6; ++i) issue(q_chunk + i + kSlots);
     q_chunk += 6;
+    // this rank's 32 dims of q, k_ae, v_ae (48 rows x 64 bytes each) to the partners
+    push_rows(qbuf + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
+    push_rows(ownk + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
+    push_rows(ownv + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
     cluster.sync();  // q, own k, own v complete in every CTA
 
     // --- Eq. 1 over keys [kbeg, kend) of [cache ; own], 32-key tiles
@@ -510,27 +546,38 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       }
     }
 
-    // --- merge the 4 splits: push each row's partial to the rank that owns it
+    // --- merge the 4 splits: stage this split's normalised partial (fp16) and
+    // log-sum-exp locally, then send each row to the rank that owns it
+    __half* part = reinterpret_cast<__half*>(tile_k);  // [48][kD] (tile area, free now)
+    float* part_lse = reinterpret_cast<float*>(smem + L.rstd);
     if (warp < 3) {
       const int qr0 = warp * 16 + (lane >> 2);
       const int qr1 = qr0 + 8;
       const float inv0 = l_run[0] > 0.f ? 1.f / l_run[0] : 0.f;
       const float inv1 = l_run[1] > 0.f ? 1.f / l_run[1] : 0.f;
-      const int own0 = qr0 / kRowsPerRank, own1 = qr1 / kRowsPerRank;
-      __half* d0 = cluster.map_shared_rank(recv, own0) + (rank * kRowsPerRank + qr0 - own0 * kRowsPerRank) * kD;
-      __half* d1 = cluster.map_shared_rank(recv, own1) + (rank * kRowsPerRank + qr1 - own1 * kRowsPerRank) * kD;
 #pragma unroll
       for (int n = 0; n < 16; ++n) {
         const int c = n * 8 + 2 * (lane & 3);
-        *reinterpret_cast<uint32_t*>(d0 + c) = pack_half2(o_acc[n][0] * inv0, o_acc[n][1] * inv0);
-        *reinterpret_cast<uint32_t*>(d1 + c) = pack_half2(o_acc[n][2] * inv1, o_acc[n][3] * inv1);
+        *reinterpret_cast<uint32_t*>(part + qr0 * kD + c) = pack_half2(o_acc[n][0] * inv0, o_acc[n][1] * inv0);
+        *reinterpret_cast<uint32_t*>(part + qr1 * kD + c) = pack_half2(o_acc[n][2] * inv1, o_acc[n][3] * inv1);
       }
       if ((lane & 3) == 0) {
-        cluster.map_shared_rank(recv_lse, own0)[rank * kRowsPerRank + qr0 - own0 * kRowsPerRank] =
-            l_run[0] > 0.f ? m_run[0] + log2f(l_run[0]) : -CUDART_INF_F;
-        cluster.map_shared_rank(recv_lse, own1)[rank * kRowsPerRank + qr1 - own1 * kRowsPerRank] =
-            l_run[1] > 0.f ? m_run[1] + log2f(l_run[1]) : -CUDART_INF_F;
+        part_lse[qr0] = l_run[0] > 0.f ? m_run[0] + log2f(l_run[0]) : -CUDART_INF_F;
+        part_lse[qr1] = l_run[1] > 0.f ? m_run[1] + log2f(l_run[1]) : -CUDART_INF_F;
       }
+    }
+    __syncthreads();
+    for (int i = tid; i < kTokTile * (kD / 8); i += kThr) {  // 48 rows x 16 units
+      const int row = i / (kD / 8);
+      const int u = i - row * (kD / 8);
+      const int owner = row / kRowsPerRank;
+      const __half* src = part + row * kD + u * 8;
+      st_cluster_v4(cluster_addr(recv + (rank * kRowsPerRank + row - owner * kRowsPerRank) * kD + u * 8, owner),
+                    *reinterpret_cast<const uint4*>(src));
+    }
+    if (tid < kTokTile) {
+      const int owner = tid / kRowsPerRank;
+      st_cluster_f32(cluster_addr(recv_lse + rank * kRowsPerRank + tid - owner * kRowsPerRank, owner), part_lse[tid]);
     }
     cluster.sync();
     // merged rows of o_h -> every partner's qbuf (now free) as the W_o input
@@ -562,15 +609,13 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         uint2 out;
         out.x = pack_half2(a0 * inv, a1 * inv);
         out.y = pack_half2(a2 * inv, a3 * inv);
-        if (row < kTokTile) {
-#pragma unroll
-          for (int dst = 0; dst < kCl; ++dst)
-            *reinterpret_cast<uint2*>(cluster.map_shared_rank(qbuf, dst) + row * kQS + c) = out;
-          if (p.attn_capture != nullptr && row < T)
-            *reinterpret_cast<uint2*>(p.attn_capture + (static_cast<size_t>(layer) * T + row) * HD + head * kD + c) = out;
-        }
+        *reinterpret_cast<uint2*>(qbuf + row * kQS + c) = out;
+        if (p.attn_capture != nullptr && row < T)
+          *reinterpret_cast<uint2*>(p.attn_capture + (static_cast<size_t>(layer) * T + row) * HD + head * kD + c) = out;
       }
     }
+    __syncthreads();
+    push_rows(qbuf + rank * kRowsPerRank * kQS, kRowsPerRank, kQS * 2, kD * 2, rank, tid, kThr);
     cluster.sync();  // o_h complete everywhere; ownk/ownv free for the transpose
 
     // --- W_o: this CTA's 128 output columns for head h (8 blocks, one per warp)
@@ -608,18 +653,15 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
           const int m = t * 8 + 2 * (lane & 3);
           const float h0 = acc[t][0] / (1.f + __expf(-acc[t][0])) * acc[t][2];
           const float h1 = acc[t][1] / (1.f + __expf(-acc[t][1])) * acc[t][3];
-#pragma unroll
-          for (int dst = 0; dst < kCl; ++dst) {
-            __half* b = cluster.map_shared_rank(hsl, dst);
-            b[m * kHS + col] = __float2half_rn(h0);
-            b[(m + 1) * kHS + col] = __float2half_rn(h1);
-          }
+          hsl[m * kHS + col] = __float2half_rn(h0);
+          hsl[(m + 1) * kHS + col] = __float2half_rn(h1);
         }
       }
       __syncthreads();
       if (tid == 0)
         for (int i = 0; i < 2; ++i) issue(q_chunk + i + kSlots);
       q_chunk += 2;
+      push_rows(hsl + rank * 16, kTokTile, kHS * 2, 32, rank, tid, kThr);
       cluster.sync();  // SwiGLU slice complete everywhere
       {
         const uint4* w = wait_chunk(q_chunk) + warp * (64 / 16) * 32;

@@ -48,7 +48,7 @@ def _cfg(**over):
 
 
 def _create(lib, cfg, weights=True):
-    w = synth.make_weights(synth.Dims(n_layers=1, d_model=64, n_heads=1, d_ff=64), 0) if weights else None
+    w = synth.make_weights(synth.Dims(n_layers=1, d_model=128, n_heads=1, d_ff=64), 0) if weights else None
     keep = None
     if weights:
         wst, keep = fsx.make_weights(w)
@@ -75,6 +75,7 @@ def test_create_rejects_null_weights(lib):
 @pytest.mark.parametrize("field,value,code", [
     ("head_dim", 64, fsx.FSX_ERR_UNSUPPORTED),
     ("d_model", 500, fsx.FSX_ERR_UNSUPPORTED),
+    ("d_model", 192, fsx.FSX_ERR_UNSUPPORTED),
     ("d_ff", 100, fsx.FSX_ERR_UNSUPPORTED),
     ("n_frame", 40, fsx.FSX_ERR_UNSUPPORTED),
     ("n_layers", 0, fsx.FSX_ERR_INVALID_ARG),
@@ -91,7 +92,7 @@ def test_create_rejects_bad_shapes(lib, field, value, code):
 
 def test_forced_allocation_failure(lib, monkeypatch):
     monkeypatch.setenv("FSX_TEST_FAIL_ALLOC", "1")
-    st, h = _create(lib, _cfg(n_layers=1, d_model=64, n_heads=1, d_ff=64))
+    st, h = _create(lib, _cfg(n_layers=1, d_model=128, n_heads=1, d_ff=64))
     assert st == fsx.FSX_ERR_OOM
     assert not h.value
 
@@ -99,7 +100,7 @@ def test_forced_allocation_failure(lib, monkeypatch):
 def test_create_without_gpu_reports_cuda_error(lib):
     if torch.cuda.is_available():
         pytest.skip("a GPU is present")
-    st, h = _create(lib, _cfg(n_layers=1, d_model=64, n_heads=1, d_ff=64))
+    st, h = _create(lib, _cfg(n_layers=1, d_model=128, n_heads=1, d_ff=64))
     assert st == fsx.FSX_ERR_CUDA
     assert not h.value
 
