@@ -31,6 +31,14 @@ UNIT = "vehicle-ticks/s"
 FALLBACK_HBM_GBS = 6800.0
 KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down", "persistent"]
 
+# DRAM bytes (read + write) of one launch of the timed kernel, from one ncu capture of the
+# kernel as it is now (profiles/ holds each summary with its command). A kernel that changed
+# after its capture gets no entry, so its traffic is reported as null.
+NCU_TRAFFIC = {
+    ("persistent", "bf16_b1_l224"): 793.065728e6 + 4.460032e6,  # persistent_tick_bf16_b1_l224.md
+    ("qkv", "bf16_b16_ragged"): 13.401088e6,                     # gemm_tc_bf16_b16_ragged.md
+}
+
 
 def parse():
     ap = argparse.ArgumentParser()
@@ -279,7 +287,7 @@ def main():
                    "parallelism": f"replicas x{world}"},
         "gpu_launches": ex.launches(B) * args.steps,
         "roofline": {"bound": "hbm", "kernel": kclass, "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": achieved / hbm, "traffic": None, "peak_source": peak_kind,
+                     "frac": achieved / hbm, "traffic": NCU_TRAFFIC.get((kclass, args.workload)), "peak_source": peak_kind,
                      "bytes_per_launch": unit_bytes, "launch_us": per_launch_s * 1e6},
         "tick_roofline": {"bytes_per_tick": tick_bytes, "kv_bytes_per_tick": kv_bytes, "achieved_gbs": tick_gbs,
                           "frac_of_measured_hbm": tick_gbs / hbm, "frac_of_8tbs": tick_gbs / 8000.0},
