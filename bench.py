@@ -35,7 +35,6 @@ KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down", "persistent"]
 # kernel as it is now (profiles/ holds each summary with its command). A kernel that changed
 # after its capture gets no entry, so its traffic is reported as null.
 NCU_TRAFFIC = {
-    ("persistent", "bf16_b1_l224"): 793.065728e6 + 4.460032e6,  # persistent_tick_bf16_b1_l224.md
     ("qkv", "bf16_b16_ragged"): 13.401088e6,                     # gemm_tc_bf16_b16_ragged.md
 }
 

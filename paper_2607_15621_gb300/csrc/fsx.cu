@@ -25,6 +25,7 @@
 #include "gemm_tc.h"
 #include "kernels.h"
 #include "persistent.h"
+#include "tcgen05.cuh"
 
 using fsx::TickArgs;
 
@@ -139,31 +140,15 @@ fsx_status check_config(const fsx_config* c) {
   return FSX_OK;
 }
 
-// fp32 -> fp16 fragment blocks of the tensor-core A operand (m16n8k16):
-// block (nb, kb) holds, for lane l, rows r = 16nb + l/4 and r + 8 and columns
-// c = 16kb + 2(l%4) (+1, +8, +9) in register order a0..a7.
+// fp32 rows -> fp16 swizzled K-major operand images of the tensor core, one
+// rows x 128-byte image per 64-wide K slice (optional per-K gain folded in)
 template <typename RowFn>
-void pack_fragments(RowFn row, int N, int K, __half* out, const float* col_scale = nullptr) {
-  const int kbs = K / 16;
-  for (int nb = 0; nb < N / 16; ++nb) {
-    for (int lane = 0; lane < 32; ++lane) {
-      const float* r0 = row(nb * 16 + (lane >> 2));
-      const float* r1 = row(nb * 16 + (lane >> 2) + 8);
-      const int c = 2 * (lane & 3);
-      for (int kb = 0; kb < kbs; ++kb) {
-        __half* o = out + ((static_cast<size_t>(nb) * kbs + kb) * 32 + lane) * 8;
-        const int k = kb * 16 + c;
-        auto sc = [&](int kk) { return col_scale ? col_scale[kk] : 1.f; };
-        o[0] = __float2half_rn(r0[k] * sc(k));
-        o[1] = __float2half_rn(r0[k + 1] * sc(k + 1));
-        o[2] = __float2half_rn(r1[k] * sc(k));
-        o[3] = __float2half_rn(r1[k + 1] * sc(k + 1));
-        o[4] = __float2half_rn(r0[k + 8] * sc(k + 8));
-        o[5] = __float2half_rn(r0[k + 9] * sc(k + 9));
-        o[6] = __float2half_rn(r1[k + 8] * sc(k + 8));
-        o[7] = __float2half_rn(r1[k + 9] * sc(k + 9));
-      }
-    }
+void pack_sw128(RowFn row, int rows, int K, const float* gain, unsigned char* out) {
+  for (int r = 0; r < rows; ++r) {
+    const float* src = row(r);
+    for (int k = 0; k < K; ++k)
+      *reinterpret_cast<__half*>(out + fsx::sw128_offset(rows, r, k)) =
+          __float2half_rn(src[k] * (gain ? gain[k] : 1.f));
   }
 }
 
@@ -581,19 +566,15 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
           const int head = cta / fsx::kPersistCluster, rank = cta % fsx::kPersistCluster;
           unsigned char* a = base + static_cast<size_t>(cta) * h->p_a_cta;
           const float* mats[3] = {w->wq + hd_d * l, w->wk + hd_d * l, w->wv + hd_d * l};
-          for (int i = 0; i < 6; ++i) {  // q, q, k, k, v, v: 16 head dims each
-            const float* m = mats[i / 2];
-            const int dim0 = head * fsx::kHeadDim + rank * 32 + (i % 2) * 16;
-            pack_fragments([&](int r) -> const float* { return m + static_cast<size_t>(dim0 + r) * d; }, 16, d,
-                           reinterpret_cast<__half*>(a + i * chunk), g1);
-          }
+          // rows 32j..32j+31: dims 32 rank .. 32 rank + 31 of head h in W_q, W_k, W_v
+          pack_sw128([&](int r) -> const float* {
+            return mats[r / 32] + static_cast<size_t>(head * fsx::kHeadDim + rank * 32 + r % 32) * d;
+          }, 96, d, g1, a);
+          // 128 output columns of this rank x this head's 128 inputs
           const float* wo = w->wo + hd_d * l;
-          for (int i = 0; i < 2; ++i) {  // 64 output columns x this head's 128 inputs
-            const int col0 = rank * 128 + i * 64;
-            pack_fragments([&](int r) -> const float* {
-              return wo + static_cast<size_t>(col0 + r) * HD + head * fsx::kHeadDim;
-            }, 64, fsx::kHeadDim, reinterpret_cast<__half*>(a + (6 + i) * chunk));
-          }
+          pack_sw128([&](int r) -> const float* {
+            return wo + static_cast<size_t>(rank * 128 + r) * HD + head * fsx::kHeadDim;
+          }, 128, fsx::kHeadDim, nullptr, a + 96 * 128 * (d / 64));  // after the 96-row QKV images
         }
         const float* wg = w->w_gate + static_cast<size_t>(F) * d * l;
         const float* wu = w->w_up + static_cast<size_t>(F) * d * l;
@@ -601,15 +582,15 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
         for (int cta = 0; cta < n_b * fsx::kPersistCluster; ++cta) {
           const int cl = cta / fsx::kPersistCluster, rank = cta % fsx::kPersistCluster;
           unsigned char* b = base + h->p_b_offset + static_cast<size_t>(cta) * h->p_b_cta;
-          for (int j = 0; j < 2; ++j) {  // 8 gate rows then the matching 8 up rows
-            const int hc0 = cl * 64 + rank * 16 + j * 8;
-            pack_fragments([&](int r) -> const float* {
-              return r < 8 ? wg + static_cast<size_t>(hc0 + r) * d : wu + static_cast<size_t>(hc0 + r - 8) * d;
-            }, 16, d, reinterpret_cast<__half*>(b + j * chunk), g2);
-          }
-          pack_fragments([&](int r) -> const float* {  // 128 output columns x this cluster's 64 SwiGLU inputs
+          // rows 0-15: gate columns 64 cl + 16 rank + r; rows 16-31: the matching up columns
+          pack_sw128([&](int r) -> const float* {
+            const int col = cl * 64 + rank * 16 + r % 16;
+            return (r < 16 ? wg : wu) + static_cast<size_t>(col) * d;
+          }, 32, d, g2, b);
+          // 128 output columns x this cluster's 64 SwiGLU inputs
+          pack_sw128([&](int r) -> const float* {
             return wd + static_cast<size_t>(rank * 128 + r) * F + cl * 64;
-          }, 128, 64, reinterpret_cast<__half*>(b + 2 * chunk));
+          }, 128, 64, nullptr, b + 32 * 128 * (d / 64));
         }
       };
       const int n_threads = std::max(1, std::min<int>(16, static_cast<int>(std::thread::hardware_concurrency())));

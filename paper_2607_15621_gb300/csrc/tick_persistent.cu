@@ -5,32 +5,40 @@
 // attention head (H clusters, 4H CTAs, one CTA per SM, all co-resident).
 // Every layer runs two phases separated by device-wide counters:
 //   phase A (every cluster = one head h):
-//     x -> RMSNorm (each CTA normalises a quarter of the rows and pushes them to
-//     its partners through distributed shared memory) -> the CTA's 96 rows of
-//     [W_q; W_k; W_v] for head h (32 q, 32 k, 32 v dims) -> q, k_ae, v_ae pushed
-//     to all 4 CTAs -> Eq. 1 over a quarter of [K_vlm ; K_ae] per CTA ->
-//     the 4 split results merged in shared memory (log-sum-exp weights) ->
-//     the CTA's 128 output columns of o_h W_o^T added into the next residual
-//     state with vector atomics (cluster 0 also adds the residual itself).
+//     x -> RMSNorm (every CTA normalises all token rows itself, straight from
+//     L2) -> the CTA's 96 rows of [W_q; W_k; W_v] for head h (32 q, 32 k, 32 v
+//     dims) on the tensor cores (tcgen05, accumulator in tensor memory) ->
+//     q, k_ae, v_ae pushed to all 4 CTAs -> Eq. 1 over a quarter of
+//     [K_vlm ; K_ae] per CTA -> the 4 split results merged in shared memory
+//     (log-sum-exp weights) -> the CTA's 128 output columns of o_h W_o^T
+//     (tcgen05) added into the next residual state with vector atomics
+//     (cluster 0 also adds the residual itself).
 //   phase B (clusters 0 .. F/64-1; cluster c owns SwiGLU columns 64c..64c+63):
-//     x -> RMSNorm (split and pushed as above) -> the CTA's 16 SwiGLU columns
-//     (gate and up rows side by side) -> h pushed to all 4 CTAs -> the CTA's
-//     128 output columns of h W_d^T added into the next residual state.
+//     x -> RMSNorm -> the CTA's 16 SwiGLU columns (16 gate rows, then the
+//     matching 16 up rows; tcgen05) -> h pushed to all 4 CTAs -> the CTA's 128
+//     output columns of h W_d^T (tcgen05) added into the next residual state.
 // The residual stream rotates through three fp32 buffers: a phase reads one,
 // accumulates into the next (zeroed one phase earlier) and zeroes the third.
 //
 // Weights never wait for activations: each CTA's weights are packed in the
-// order it consumes them (16 KB chunks, fragment-ordered fp16) and streamed by
-// bulk copies through a 6-slot shared-memory ring that is refilled as soon as
-// a chunk is consumed, so the HBM stream runs ahead across phases and layers.
-// The layer's backbone cache rows are prefetched into L2 at the start of the
-// layer and converted bf16/fp32 -> fp16 while staging 32-key tiles.
+// order it consumes them, as the swizzled K-major images the tensor core reads
+// (128-byte swizzle, one 64-wide K slice per image), and streamed by bulk
+// copies through a 6-slot ring of 16 KB that is refilled as soon as a GEMM has
+// finished with its slots, so the HBM stream runs ahead across phases and
+// layers. A layer takes 12 ring positions (6 of QKV, 2 of W_o, 2 of gate/up,
+// 1 of W_d and one empty position; CTAs without SwiGLU work leave positions
+// 8-11 empty), so the QKV images of every layer start at slot 0. The MMAs run
+// with M = 128: the 96-row QKV and 32-row gate/up images are padded with
+// whatever follows them in shared memory, and the rows that produces are never
+// read. The layer's backbone cache rows are prefetched into L2 at the start of
+// the layer and converted bf16/fp32 -> fp16 while staging 32-key tiles.
 #include <cooperative_groups.h>
 #include <math_constants.h>
 
 #include "device_util.cuh"
 #include "kernels.h"
 #include "persistent.h"
+#include "tcgen05.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -42,38 +50,44 @@ constexpr int kThr = kPersistThreads;  // 256 = 8 warps
 constexpr int kCl = kPersistCluster;   // 4 CTAs per cluster
 constexpr int kSlotBytes = kPersistChunk;
 constexpr int kSlots = kPersistSlots;
+constexpr int kLayerChunks = 2 * kSlots;      // ring positions per layer, empty ones included
 constexpr int kD = kHeadDim;           // 128
 constexpr int kKeyTile = 32;           // keys per staged attention tile
-constexpr int kQS = kD + 8;            // fp16 row stride of q / own k / own v / o (halves)
-constexpr int kHS = 64 + 8;            // fp16 row stride of the SwiGLU slice (halves)
+constexpr int kQS = kD + 8;            // fp16 row stride of q / own k / own v (halves)
 constexpr int kDS = 128 + 4;           // fp32 row stride of the output transpose buffer
 constexpr int kRowsPerRank = kTokTile / kCl;  // 12
+constexpr int kQkvAtom = 3 * 32 * 128;        // one 64-wide K slice of the CTA's 96 QKV rows (12 KB)
+constexpr int kGuAtom = 32 * 128;             // one K slice of the 32 gate/up rows (4 KB)
+constexpr int kActAtom = kTokTile * 128;      // one K slice of the 48 token rows (6 KB)
+constexpr uint32_t kTmemCols = 64;            // accumulator: 128 lanes x 48 fp32 columns
+constexpr uint32_t kIdesc = idesc_f16(128, kTokTile);
 constexpr unsigned long long kSpinLimitNs = 1000000000ull;
+#ifndef FSX_NORM_BATCH
+#define FSX_NORM_BATCH 2
+#endif
 
 struct Smem {
-  // byte offsets inside the dynamic shared memory
-  int full_bar, rstd, ring, act, qbuf, ownk, ownv, tile, recv, recv_lse, total;
+  // byte offsets from the 1024-byte aligned base of the dynamic shared memory
+  int bars, lse, ring, act, qbuf, ownk, ownv, tile, recv, recv_lse, total;
 };
 
 __host__ __device__ inline Smem smem_layout(int d) {
   Smem s{};
-  int o = 0;
-  s.full_bar = o;  o += 64;
-  s.rstd = o;      o += 256;
-  o = 1024;
-  s.ring = o;      o += kSlots * kSlotBytes;
-  s.act = o;       o += kTokTile * (d + 8) * 2;
-  s.qbuf = o;      o += kTokTile * kQS * 2;            // q of this head; later the merged o_h
-  s.ownk = o;      o += kTokTile * kQS * 2;            // own keys; later the output transpose
-  s.ownv = o;      o += kTokTile * kQS * 2;            // own values
-  s.tile = o;      o += 2 * kKeyTile * kD * 2;         // fp16 K|V tile, swizzled
-  s.recv = o;      o += kCl * kRowsPerRank * kD * 2;   // fp16 split partials of the rows this CTA merges
+  s.bars = 0;                                  // ring barriers, MMA barrier, TMEM address
+  s.lse = 256;                                 // [48] fp32 log-sum-exp of this split
+  int o = 1024;
+  s.ring = o;      o += kSlots * kSlotBytes;   // also read 4 KB past its end by the last QKV MMA
+  s.act = o;       o += (d / 64) * kActAtom;   // normalised x, swizzled (B operand of QKV, gate/up)
+  s.qbuf = o;      o += kTokTile * kQS * 2;    // q of this head; in phase B the swizzled SwiGLU slice
+  s.ownk = o;      o += kTokTile * kQS * 2;    // own keys; later the output transpose
+  s.ownv = o;      o += kTokTile * kQS * 2;    // own values
+  o = (o + 1023) & ~1023;
+  s.tile = o;      o += 2 * kKeyTile * kD * 2; // fp16 K|V tile; later the merged o_h, swizzled
+  s.recv = o;      o += kCl * kRowsPerRank * kD * 2;  // fp16 split partials of the rows this CTA merges
   s.recv_lse = o;  o += kCl * kRowsPerRank * 4;
-  s.total = o;
+  s.total = o + 1024;                          // + alignment slack of the dynamic base
   return s;
 }
-
-__device__ __forceinline__ int swz(int row, int unit) { return row * 16 + (unit ^ (row & 7)); }
 
 __device__ __forceinline__ float4 ld_cg4(const float* p) { return __ldcg(reinterpret_cast<const float4*>(p)); }
 
@@ -126,10 +140,10 @@ __device__ __forceinline__ void push_rows(const void* base, int rows, int row_st
 }
 
 // Bounded wait until *counter >= target (one thread polls, the CTA follows).
-// Once any wait of the tick has timed out, later waits return immediately, so
-// a broken tick still ends within about a second.
-__device__ __forceinline__ void wait_counter(const int* counter, int target, int* status) {
-  if (threadIdx.x == 0 && *reinterpret_cast<volatile int*>(status) != kStatusTimeout) {
+// Once a wait of this CTA has timed out (*abort set), later waits return at
+// once, so a broken tick still ends within about a second per CTA.
+__device__ __forceinline__ void wait_counter(const int* counter, int target, int* status, volatile int* abort) {
+  if (threadIdx.x == 0 && *abort == 0) {
     const unsigned long long t0 = global_timer_ns();
     for (uint32_t it = 0;; ++it) {
       int v;
@@ -137,6 +151,7 @@ __device__ __forceinline__ void wait_counter(const int* counter, int target, int
       if (v >= target) break;
       if ((it & 63u) == 63u && global_timer_ns() - t0 > kSpinLimitNs) {
         set_status(status, kStatusTimeout);
+        *abort = 1;
         break;
       }
     }
@@ -144,42 +159,23 @@ __device__ __forceinline__ void wait_counter(const int* counter, int target, int
   __syncthreads();
 }
 
-// One 16-row weight block (fragment-ordered, kbs k-steps of 16) against the
-// 48-token activation tile `act` (row stride `as` halves): acc[token tile][4].
-__device__ __forceinline__ void block_gemm(const uint4* w, int kbs, const __half* act, int as, float (&acc)[6][4],
-                                           int lane) {
-#pragma unroll
-  for (int t = 0; t < 6; ++t)
-#pragma unroll
-    for (int e = 0; e < 4; ++e) acc[t][e] = 0.f;
-  for (int kb = 0; kb < kbs; kb += 2) {
-    uint32_t b[6][2][2];
-#pragma unroll
-    for (int t = 0; t < 6; ++t) {
-      const __half* src = act + static_cast<size_t>(t * 8 + (lane & 7)) * as + kb * 16 + (lane >> 3) * 8;
-      ldsm_x4(b[t][0][0], b[t][0][1], b[t][1][0], b[t][1][1], smem_addr(src));
-    }
-#pragma unroll
-    for (int kk = 0; kk < 2; ++kk) {
-      const uint4 a = w[(kb + kk) * 32 + lane];
-#pragma unroll
-      for (int t = 0; t < 6; ++t) mma_f16_16816(acc[t], a.x, a.y, a.z, a.w, b[t][kk][0], b[t][kk][1]);
-    }
-  }
-}
-
 template <typename CT>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persistent_tick_kernel(const PersistArgs p) {
-  extern __shared__ __align__(1024) unsigned char smem[];
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  // the swizzled operand images need 1024-byte aligned shared addresses
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const Smem L = smem_layout(p.d);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.full_bar);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bars);
+  uint64_t* mma_bar = full + kSlots;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_bar + 1);
   unsigned char* ring = smem + L.ring;
-  __half* act = reinterpret_cast<__half*>(smem + L.act);
+  unsigned char* act = smem + L.act;
   __half* qbuf = reinterpret_cast<__half*>(smem + L.qbuf);
   __half* ownk = reinterpret_cast<__half*>(smem + L.ownk);
   __half* ownv = reinterpret_cast<__half*>(smem + L.ownv);
-  uint4* tile_k = reinterpret_cast<uint4*>(smem + L.tile);
-  uint4* tile_v = tile_k + kKeyTile * 16;
+  unsigned char* hsl = smem + L.qbuf;  // phase B: swizzled [48 tokens x 64] SwiGLU slice of the cluster
+  unsigned char* obuf = smem + L.tile;  // merged o_h, swizzled [48 tokens x 128]
   __half* recv = reinterpret_cast<__half*>(smem + L.recv);
   float* recv_lse = reinterpret_cast<float*>(smem + L.recv_lse);
   float* dstT = reinterpret_cast<float*>(smem + L.ownk);  // [48][kDS] fp32 output transpose (aliases ownk/ownv)
@@ -192,36 +188,57 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   const int head = blockIdx.x / kCl;             // phase A: this cluster's head
   const int G = gridDim.x;
   const int cta = blockIdx.x;
-  const int d = p.d;
-  const int as = d + 8;
+  const int d = p.d;                             // 512 (checked on the host)
   const int T = p.n_action + p.n_frame;
   const int HD = p.H * kD;
   const bool in_b = head < p.n_b_clusters;       // phase B participant (whole clusters)
   const int n_b_ctas = p.n_b_clusters * kCl;
-  const int per_layer = kPersistAChunks + (in_b ? kPersistBChunks : 0);
-  const int total_chunks = p.n_layers * per_layer;
+  const int total_chunks = p.n_layers * kLayerChunks;
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + L.bars + 96);  // a wait of this CTA timed out
 
-  // ---- ring: chunk q of this CTA's stream goes to slot q % kSlots
+  // ---- ring: position q of this CTA's stream uses slot q % kSlots; per layer
+  // positions 0-7 are phase-A images, 8-10 phase-B images, the rest empty
   auto chunk_src = [&](int q) -> const unsigned char* {
-    const int layer = q / per_layer;
-    const int i = q - layer * per_layer;
+    const int layer = q / kLayerChunks;
+    const int i = q - layer * kLayerChunks;
     const unsigned char* base = p.warena + static_cast<size_t>(layer) * p.layer_bytes;
     if (i < kPersistAChunks) return base + static_cast<size_t>(cta) * p.a_cta_bytes + static_cast<size_t>(i) * kSlotBytes;
-    return base + p.b_offset + static_cast<size_t>(cta) * p.b_cta_bytes + static_cast<size_t>(i - kPersistAChunks) * kSlotBytes;
+    return base + p.b_offset + static_cast<size_t>(cta) * p.b_cta_bytes +
+           static_cast<size_t>(i - kPersistAChunks) * kSlotBytes;
   };
-  auto issue = [&](int q) {  // called by thread 0 only
+  auto is_empty = [&](int q) {
+    const int i = q % kLayerChunks;
+    return i >= kPersistAChunks + (in_b ? kPersistBChunks : 0);
+  };
+  auto issue = [&](int q) {  // one thread; an empty position just completes the slot's phase
     if (q >= total_chunks) return;
     uint64_t* bar = full + (q % kSlots);
+    if (is_empty(q)) {
+      mbar_arrive(bar);
+      return;
+    }
     mbar_arrive_expect_tx(bar, kSlotBytes);
     bulk_g2s(ring + static_cast<size_t>(q % kSlots) * kSlotBytes, chunk_src(q), kSlotBytes, bar);
   };
-  auto wait_chunk = [&](int q) -> const uint4* {
-    mbar_wait(full + (q % kSlots), static_cast<uint32_t>((q / kSlots) & 1), p.status);
-    return reinterpret_cast<const uint4*>(ring + static_cast<size_t>(q % kSlots) * kSlotBytes);
+  // wait for position q; false after a timeout of this tick (no MMA then reads the slot)
+  auto wait_chunk = [&](int q) -> bool {
+    if (*abort) return false;
+    const bool ok = mbar_wait(full + (q % kSlots), static_cast<uint32_t>((q / kSlots) & 1), p.status);
+    if (!ok) *abort = 1;
+    return ok;
+  };
+  uint32_t n_mma = 0;  // completed MMA groups (phase of mma_bar)
+  // all threads: wait for the MMA group just committed, then order TMEM reads after it
+  auto wait_mma = [&]() {
+    if (*abort == 0 && !mbar_wait(mma_bar, n_mma & 1u, p.status)) *abort = 1;
+    ++n_mma;
+    tc_fence_after();
   };
 
   if (tid == 0) {
+    *abort = 0;
     for (int i = 0; i < kSlots; ++i) mbar_init(full + i, 1);
+    mbar_init(mma_bar, 1);
     for (int q = 0; q < kSlots; ++q) issue(q);
   }
 
@@ -236,9 +253,31 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   __syncthreads();
   if (bad) {
     if (cta == 0 && tid == 0) set_status(p.status, kStatusDeviceArg);
-    for (int q = 0; q < kSlots && q < total_chunks; ++q) wait_chunk(q);  // let in-flight copies land
+    if (tid == 0)
+      for (int q = 0; q < kSlots && q < total_chunks; ++q) wait_chunk(q);  // let in-flight copies land
     return;
   }
+
+  // ---- tensor memory for the accumulator (one CTA per SM: never contended)
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(tmem_slot)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  // token rows T..47 of the activation image stay zero for the whole tick
+  for (int i = tid; i < (kTokTile - T) * (d / 8); i += kThr) {
+    const int r = T + i / (d / 8);
+    const int k = (i % (d / 8)) * 8;
+    *reinterpret_cast<uint4*>(act + sw128_offset(kTokTile, r, k)) = make_uint4(0u, 0u, 0u, 0u);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(tmem_slot);
+  const uint32_t ring_a = smem_addr(ring);
+  const uint32_t act_a = smem_addr(act);
+
   const long long Lc = o_hi - o_lo;
   const long long n_keys = Lc + T;
   const long long kbeg = n_keys * rank / kCl;
@@ -269,48 +308,52 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   }
   arrive(p.counters + 0);
 
-  // x (state buffer) -> RMSNorm -> fp16 rows in every partner's activation tile:
-  // this rank normalises rows 12r..12r+11 into its own tile and copies them out
+  // x (state buffer in L2) -> RMSNorm -> fp16 rows of the swizzled activation
+  // image. Warp w takes rows w, w+8, ... (rotated by 8 (cta mod 6), so that the
+  // 128 CTAs reading the same 84 KB spread over all rows at any moment instead of
+  // queueing on the same L2 lines); lane l takes columns 16l..16l+15. Every load
+  // of the warp is issued before the first use: one L2 round trip covers all.
+  const int row_rot = (cta % 6) * 8;
   auto load_normalized = [&](const float* Xs) {
-    const int r0 = rank * kRowsPerRank;
-    const int r1 = min(r0 + kRowsPerRank, T);
-    for (int r = r0 + warp; r < r1; r += kThr / 32) {
-      const float* xr = Xs + static_cast<size_t>(r) * d;
-      float4 v[8];
-      float ss = 0.f;
+    constexpr int kRowsPerWarp = kTokTile / (kThr / 32);  // 6
+    constexpr int kBatch = FSX_NORM_BATCH;                // rows in flight per warp
+#pragma unroll 1
+    for (int i0 = 0; i0 < kRowsPerWarp; i0 += kBatch) {
+      float4 v[kBatch][4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {  // lane holds 8 consecutive values per 256-wide slab
-        const int c = lane * 8 + j * 256;
-        if (c < d) {
-          v[2 * j] = ld_cg4(xr + c);
-          v[2 * j + 1] = ld_cg4(xr + c + 4);
-          ss += v[2 * j].x * v[2 * j].x + v[2 * j].y * v[2 * j].y + v[2 * j].z * v[2 * j].z + v[2 * j].w * v[2 * j].w;
-          ss += v[2 * j + 1].x * v[2 * j + 1].x + v[2 * j + 1].y * v[2 * j + 1].y + v[2 * j + 1].z * v[2 * j + 1].z +
-                v[2 * j + 1].w * v[2 * j + 1].w;
+      for (int i = 0; i < kBatch; ++i) {
+        const int r = (warp + 8 * (i0 + i) + row_rot) % kTokTile;
+        if (r < T) {
+          const float* xr = Xs + static_cast<size_t>(r) * d + lane * 16;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) v[i][j] = ld_cg4(xr + 4 * j);
         }
       }
-      ss = warp_sum(ss);
-      const float rstd = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int c = lane * 8 + j * 256;
-        if (c < d) {
-          uint4 pk;
-          pk.x = pack_half2(v[2 * j].x * rstd, v[2 * j].y * rstd);
-          pk.y = pack_half2(v[2 * j].z * rstd, v[2 * j].w * rstd);
-          pk.z = pack_half2(v[2 * j + 1].x * rstd, v[2 * j + 1].y * rstd);
-          pk.w = pack_half2(v[2 * j + 1].z * rstd, v[2 * j + 1].w * rstd);
-          *reinterpret_cast<uint4*>(act + static_cast<size_t>(r) * as + c) = pk;
+      for (int i = 0; i < kBatch; ++i) {
+        const int r = (warp + 8 * (i0 + i) + row_rot) % kTokTile;
+        if (r < T) {
+          float ss = 0.f;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) ss += v[i][j].x * v[i][j].x + v[i][j].y * v[i][j].y + v[i][j].z * v[i][j].z + v[i][j].w * v[i][j].w;
+          ss = warp_sum(ss);
+          const float rstd = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
+          uint4 lo, hi;
+          lo.x = pack_half2(v[i][0].x * rstd, v[i][0].y * rstd);
+          lo.y = pack_half2(v[i][0].z * rstd, v[i][0].w * rstd);
+          lo.z = pack_half2(v[i][1].x * rstd, v[i][1].y * rstd);
+          lo.w = pack_half2(v[i][1].z * rstd, v[i][1].w * rstd);
+          hi.x = pack_half2(v[i][2].x * rstd, v[i][2].y * rstd);
+          hi.y = pack_half2(v[i][2].z * rstd, v[i][2].w * rstd);
+          hi.z = pack_half2(v[i][3].x * rstd, v[i][3].y * rstd);
+          hi.w = pack_half2(v[i][3].z * rstd, v[i][3].w * rstd);
+          *reinterpret_cast<uint4*>(act + sw128_offset(kTokTile, r, lane * 16)) = lo;
+          *reinterpret_cast<uint4*>(act + sw128_offset(kTokTile, r, lane * 16 + 8)) = hi;
         }
       }
     }
-    for (int i = tid; i < (kTokTile - T) * (d / 8); i += kThr) {  // padding token rows
-      const int r = T + i / (d / 8);
-      *reinterpret_cast<uint4*>(act + static_cast<size_t>(r) * as + (i % (d / 8)) * 8) = make_uint4(0u, 0u, 0u, 0u);
-    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // visible to the tensor core
     __syncthreads();
-    if (r1 > r0) push_rows(act + static_cast<size_t>(r0) * as, r1 - r0, as * 2, d * 2, rank, tid, kThr);
-    cluster.sync();
   };
 
   // add the CTA's [48 x 128] transposed output (dstT) into X_next columns col0..col0+127,
@@ -331,24 +374,109 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     }
   };
 
-  // acc (16-row block x 48 tokens) -> dstT rows = tokens, columns col..col+15
-  auto store_transposed = [&](const float (&acc)[6][4], int col) {
+  // accumulator (128 output columns x 48 tokens) -> dstT[token][column]; warps
+  // 0-3 take tokens 0-31, warps 4-7 tokens 32-47 of their 32 TMEM lanes
+  auto tmem_to_dstT = [&]() {
+    const int col = (warp & 3) * 32 + lane;
+    const uint32_t taddr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+    for (int c0 = warp < 4 ? 0 : 32; c0 < (warp < 4 ? 32 : 48); c0 += 16) {
+      float v[16];
+      __syncwarp();
+      tmem_ld16(taddr + static_cast<uint32_t>(c0), v);
 #pragma unroll
-    for (int t = 0; t < 6; ++t) {
-      const int m = t * 8 + 2 * (lane & 3);
-      const int n = col + (lane >> 2);
-      dstT[m * kDS + n] = acc[t][0];
-      dstT[(m + 1) * kDS + n] = acc[t][1];
-      dstT[m * kDS + n + 8] = acc[t][2];
-      dstT[(m + 1) * kDS + n + 8] = acc[t][3];
+      for (int j = 0; j < 16; ++j) dstT[(c0 + j) * kDS + col] = v[j];
     }
+    tc_fence_before();
+    __syncthreads();
   };
 
-  int q_chunk = 0;  // next chunk of this CTA's stream to consume
-  const float scale_log2 = 1.4426950408889634f * rsqrtf(static_cast<float>(kD));
-  const size_t cache_row = static_cast<size_t>(p.H) * kD;  // elements between consecutive tokens
+  // one K slice (4 MMAs of K = 16) of D[128 x 48] (+)= A[128 rows] . B[48 tokens]^T
+  auto mma_slice = [&](uint32_t a_addr, uint32_t b_addr, bool first) {
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk)
+      umma_f16(tmem, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32), kIdesc,
+               (first && kk == 0) ? 0u : 1u);
+  };
 
-  for (int layer = 0; layer < p.n_layers; ++layer) {
+  // ---- this CTA's cache rows of a layer, staged in the activation image (free
+  // from the end of the QKV MMA to the next RMSNorm): two halves of kStageKeys
+  // keys, K rows then V rows, each row padded to kRowStride bytes so ldmatrix
+  // reads are conflict-free. Rows arrive raw (bf16 / fp32) by 16-byte cp.async
+  // copies spread over all threads and are converted to fp16 in place (at the
+  // start of the row).
+  constexpr int kRowStride = sizeof(CT) == 2 ? kD * 2 + 16 : kD * 4 + 16;  // 272 / 528 bytes
+  constexpr int kHalfBytes = 8 * kActAtom / 2;                            // 24 KB (d = 512)
+  constexpr int kStageKeys = kHalfBytes / (2 * kRowStride);               // 45 / 23 keys
+  const long long c_hi = min(kend, Lc);
+  const int n_cache = c_hi > kbeg ? static_cast<int>(c_hi - kbeg) : 0;  // cache keys of this CTA
+  const int n_chunks = (n_cache + kStageKeys - 1) / kStageKeys;
+  const int own_lo = static_cast<int>(max(kbeg, Lc) - Lc);              // own keys of this CTA
+  const int own_n = static_cast<int>(kend - Lc) - own_lo;
+  // all threads: 16-byte cp.async copies of chunk j into half j & 1 (one commit group)
+  constexpr int kUnitsPerRow = kD * static_cast<int>(sizeof(CT)) / 16;  // 16 / 32
+  auto stage_issue = [&](int j, const CT* kc, const CT* vc) {
+    const int k0 = j * kStageKeys;
+    const int n = min(kStageKeys, n_cache - k0);
+    unsigned char* kb = act + (j & 1) * kHalfBytes;
+    for (int i = tid; i < 2 * n * kUnitsPerRow; i += kThr) {  // (K|V, key, unit)
+      const int kv = i / (n * kUnitsPerRow);
+      const int rest = i - kv * n * kUnitsPerRow;
+      const int key = rest / kUnitsPerRow;
+      const int u = rest - key * kUnitsPerRow;
+      const unsigned char* src = reinterpret_cast<const unsigned char*>(kv ? vc : kc) +
+                                 ((static_cast<size_t>(o_lo + kbeg + k0 + key) * p.H + head) * kD) * sizeof(CT) + u * 16;
+      cp_async_16(smem_addr(kb + kv * kStageKeys * kRowStride + key * kRowStride + u * 16), src);
+    }
+    cp_async_commit();
+  };
+  // all threads: wait for chunk j and convert it to fp16 in place
+  auto stage_ready = [&](int j) {
+    const int h = j & 1;
+    if (j + 1 < n_chunks)  // chunk j + 1 is the only younger group in flight
+      cp_async_wait<1>();
+    else
+      cp_async_wait<0>();
+    __syncthreads();
+    const int n = min(kStageKeys, n_cache - j * kStageKeys);
+    unsigned char* kb = act + h * kHalfBytes;
+    if (sizeof(CT) == 2) {
+      for (int i = tid; i < 2 * n * 16; i += kThr) {  // (K|V, key, 16-byte unit)
+        const int kv = i / (n * 16);
+        const int rest = i - kv * n * 16;
+        uint4* ptr = reinterpret_cast<uint4*>(kb + kv * kStageKeys * kRowStride + (rest >> 4) * kRowStride + (rest & 15) * 16);
+        const uint4 raw = *ptr;
+        *ptr = make_uint4(bf16x2_to_half2(raw.x), bf16x2_to_half2(raw.y), bf16x2_to_half2(raw.z), bf16x2_to_half2(raw.w));
+      }
+    } else {
+      // 32-byte fp32 unit u of a row -> 16-byte fp16 unit u at the row start: all reads
+      // of a round land before its writes, and a unit's input is never written by a
+      // later round
+      for (int base = 0; base < 2 * n * 16; base += kThr) {
+        const int i = base + tid;
+        uint4 o = make_uint4(0u, 0u, 0u, 0u);
+        unsigned char* row = nullptr;
+        int u = 0;
+        if (i < 2 * n * 16) {
+          const int kv = i / (n * 16);
+          const int rest = i - kv * n * 16;
+          row = kb + kv * kStageKeys * kRowStride + (rest >> 4) * kRowStride;
+          u = rest & 15;
+          const float4 a = *reinterpret_cast<const float4*>(row + u * 32);
+          const float4 b = *reinterpret_cast<const float4*>(row + u * 32 + 16);
+          o = make_uint4(pack_half2(a.x, a.y), pack_half2(a.z, a.w), pack_half2(b.x, b.y), pack_half2(b.z, b.w));
+        }
+        __syncthreads();
+        if (row != nullptr) *reinterpret_cast<uint4*>(row + u * 16) = o;
+        __syncthreads();
+      }
+    }
+    __syncthreads();
+  };
+
+  int q0 = 0;  // first ring position of the current layer
+  const float scale_log2 = 1.4426950408889634f * rsqrtf(static_cast<float>(kD));
+
+  for (int layer = 0; layer < p.n_layers; ++layer, q0 += kLayerChunks) {
     const int sA = 2 * layer;
     float* Xc = X0 + static_cast<size_t>(sA % 3) * xs;        // layer input
     float* Xm = X0 + static_cast<size_t>((sA + 1) % 3) * xs;  // after attention
@@ -367,7 +495,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     }
 
     // =========================== phase A ===========================
-    wait_counter(p.counters + sA, sA == 0 ? G : n_b_ctas, p.status);
+    wait_counter(p.counters + sA, sA == 0 ? G : n_b_ctas, p.status, abort);
     // zero the buffer phase B accumulates into
     {
       const int e0 = static_cast<int>(static_cast<long long>(n_elem) * cta / G);
@@ -376,110 +504,84 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     }
     load_normalized(Xc);
 
-    // --- QKV: 6 blocks (q dims 32r..32r+31, then k, then v), one warp each
-    if (warp < 6) {
-      const uint4* w = wait_chunk(q_chunk + warp);
-      float acc[6][4];
-      block_gemm(w, d / 16, act, as, acc, lane);
-      const int kind = warp >> 1;                       // 0 q, 1 k, 2 v
-      const int dim = rank * 32 + (warp & 1) * 16 + (lane >> 2);
+    // --- QKV: D[96 (+32 unused) rows x 48 tokens] over K = 512; the 12 KB K
+    // slices lie back to back in slots 0-5, so slice a needs the slots it touches
+    if (warp == 0) {
+      tc_fence_after();
+      bool ok = true;
+      int waited = -1;
+      for (int a = 0; a < d / 64; ++a) {
+        const int last = (a * kQkvAtom + kQkvAtom - 1) / kSlotBytes;
+        while (waited < last) ok = wait_chunk(q0 + ++waited) && ok;
+        if (ok && lane == 0) mma_slice(ring_a + a * kQkvAtom, act_a + a * kActAtom, a == 0);
+        __syncwarp();
+      }
+      if (lane == 0) umma_commit(mma_bar);
+      __syncwarp();
+    }
+    wait_mma();
+    for (int j = 0; j < 2 && j < n_chunks; ++j)  // the activation image is free: stage the cache rows
+      stage_issue(j, kc, vc);
+    // rows 32j..32j+31 of the accumulator are q, k, v dims 32 rank .. 32 rank + 31
+    if ((warp & 3) < 3) {
+      const int kind = warp & 3;
       __half* b = kind == 0 ? qbuf : (kind == 1 ? ownk : ownv);
+      const int dim = rank * 32 + lane;
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(kind * 32) << 16);
+      for (int c0 = warp < 4 ? 0 : 32; c0 < (warp < 4 ? 32 : 48); c0 += 16) {
+        float v[16];
+        __syncwarp();
+        tmem_ld16(taddr + static_cast<uint32_t>(c0), v);
 #pragma unroll
-      for (int t = 0; t < 6; ++t) {
-        const int m = t * 8 + 2 * (lane & 3);
-        b[m * kQS + dim] = __float2half_rn(acc[t][0]);
-        b[(m + 1) * kQS + dim] = __float2half_rn(acc[t][1]);
-        b[m * kQS + dim + 8] = __float2half_rn(acc[t][2]);
-        b[(m + 1) * kQS + dim + 8] = __float2half_rn(acc[t][3]);
+        for (int j = 0; j < 16; ++j) b[(c0 + j) * kQS + dim] = __float2half_rn(v[j]);
       }
     }
+    tc_fence_before();
     __syncthreads();
-    if (tid == 0)
-      for (int i = 0; i < 6; ++i) issue(q_chunk + i + kSlots);
-    q_chunk += 6;
+    if (tid == 0)  // slots 0-5 are free: W_o, gate/up, W_d of this layer
+      for (int i = kSlots; i < kLayerChunks; ++i) issue(q0 + i);
     // this rank's 32 dims of q, k_ae, v_ae (48 rows x 64 bytes each) to the partners
     push_rows(qbuf + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
     push_rows(ownk + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
     push_rows(ownv + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
     cluster.sync();  // q, own k, own v complete in every CTA
 
-    // --- Eq. 1 over keys [kbeg, kend) of [cache ; own], 32-key tiles
-    float o_acc[16][4];
+    // --- Eq. 1 over keys [kbeg, kend) of [cache ; own] in 32-key tiles. Warp w < 6
+    // takes query rows 16 (w % 3) .. +15 and value dims 64 (w / 3) .. +63; both
+    // warps of a query tile compute the full scores, so no in-CTA merge is needed.
+    const int qt = warp % 3;
+    const int dh = warp / 3;
+    float o_acc[8][4];
     float m_run[2] = {-CUDART_INF_F, -CUDART_INF_F};
     float l_run[2] = {0.f, 0.f};
 #pragma unroll
-    for (int n = 0; n < 16; ++n)
+    for (int n = 0; n < 8; ++n)
 #pragma unroll
       for (int e = 0; e < 4; ++e) o_acc[n][e] = 0.f;
     uint32_t qf[8][4];
-    if (warp < 3) {
+    if (warp < 6) {
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
-        const __half* src = qbuf + static_cast<size_t>(warp * 16 + (lane & 15)) * kQS + kk * 16 + (lane >> 4) * 8;
+        const __half* src = qbuf + static_cast<size_t>(qt * 16 + (lane & 15)) * kQS + kk * 16 + (lane >> 4) * 8;
         ldsm_x4(qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3], smem_addr(src));
       }
     }
-    const int n_tiles = kend > kbeg ? static_cast<int>((kend - kbeg + kKeyTile - 1) / kKeyTile) : 0;
-    // each thread stages 4 of the 1024 16-byte units (K|V x 32 rows x 16 units) of a tile
-    uint4 stage[4];
-    auto load_tile = [&](int ti) {
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int u = tid + j * kThr;            // 0..1023
-        const int kv = u >> 9;                   // 0 = K, 1 = V
-        const int r = (u >> 4) & 31;
-        const int c = u & 15;
-        const long long key = kbeg + static_cast<long long>(ti) * kKeyTile + r;
-        uint4 val = make_uint4(0u, 0u, 0u, 0u);
-        if (key < kend) {
-          if (key < Lc) {
-            const CT* src = (kv ? vc : kc) + (static_cast<size_t>(o_lo + key) * p.H + head) * kD + c * 8;
-            if (sizeof(CT) == 2) {
-              const uint4 raw = __ldg(reinterpret_cast<const uint4*>(src));
-              val = make_uint4(bf16x2_to_half2(raw.x), bf16x2_to_half2(raw.y), bf16x2_to_half2(raw.z),
-                               bf16x2_to_half2(raw.w));
-            } else {
-              const float4 a = __ldg(reinterpret_cast<const float4*>(src));
-              const float4 b = __ldg(reinterpret_cast<const float4*>(src) + 1);
-              val = make_uint4(pack_half2(a.x, a.y), pack_half2(a.z, a.w), pack_half2(b.x, b.y), pack_half2(b.z, b.w));
-            }
-          } else {
-            const __half* own = (kv ? ownv : ownk) + static_cast<size_t>(key - Lc) * kQS + c * 8;
-            val = *reinterpret_cast<const uint4*>(own);
-          }
-        }
-        stage[j] = val;
-      }
-    };
-    auto store_tile = [&]() {
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int u = tid + j * kThr;
-        const int kv = u >> 9;
-        const int r = (u >> 4) & 31;
-        const int c = u & 15;
-        (kv ? tile_v : tile_k)[swz(r, c)] = stage[j];
-      }
-    };
-    (void)cache_row;
-    if (n_tiles > 0) {
-      load_tile(0);
-      store_tile();
-    }
-    __syncthreads();
-    for (int ti = 0; ti < n_tiles; ++ti) {
-      if (ti + 1 < n_tiles) load_tile(ti + 1);  // in flight while the tile is consumed
-      if (warp < 3) {
-        const int rows = static_cast<int>(min(static_cast<long long>(kKeyTile), kend - kbeg - static_cast<long long>(ti) * kKeyTile));
+    // keys 0..n-1 with K rows at kb and V rows at vb (fp16, `stride` bytes apart)
+    auto attend = [&](const unsigned char* kb, const unsigned char* vb, int stride, int n) {
+      for (int t0 = 0; t0 < n; t0 += kKeyTile) {
+        const int rows = min(kKeyTile, n - t0);
         float sc[4][4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
 #pragma unroll
           for (int e = 0; e < 4; ++e) sc[j][e] = 0.f;
+          int r = t0 + j * 8 + (lane & 7);
+          r = r < n ? r : 0;  // masked below; any valid row keeps the products finite
+          const uint32_t krow = smem_addr(kb + r * stride);
 #pragma unroll
           for (int dd = 0; dd < 4; ++dd) {
             uint32_t b0, b1, b2, b3;
-            ldsm_x4(b0, b1, b2, b3, smem_addr(tile_k + swz(j * 8 + (lane & 7), dd * 4 + (lane >> 3))));
+            ldsm_x4(b0, b1, b2, b3, krow + (dd * 4 + (lane >> 3)) * 16);
             mma_f16_16816(sc[j], qf[2 * dd][0], qf[2 * dd][1], qf[2 * dd][2], qf[2 * dd][3], b0, b1);
             mma_f16_16816(sc[j], qf[2 * dd + 1][0], qf[2 * dd + 1][1], qf[2 * dd + 1][2], qf[2 * dd + 1][3], b2, b3);
           }
@@ -521,7 +623,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
           l_run[r] = l_run[r] * alpha[r] + rs[r];
         }
 #pragma unroll
-        for (int n = 0; n < 16; ++n) {
+        for (int n = 0; n < 8; ++n) {
           o_acc[n][0] *= alpha[0];
           o_acc[n][1] *= alpha[0];
           o_acc[n][2] *= alpha[1];
@@ -529,39 +631,48 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         }
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
+          int r = t0 + kk * 16 + (lane & 7) + 8 * ((lane >> 3) & 1);
+          r = r < n ? r : 0;
+          const uint32_t vrow = smem_addr(vb + r * stride);
 #pragma unroll
-          for (int np = 0; np < 8; ++np) {
+          for (int np = 0; np < 4; ++np) {
             uint32_t b0, b1, b2, b3;
-            ldsm_x4_trans(b0, b1, b2, b3,
-                          smem_addr(tile_v + swz(kk * 16 + (lane & 7) + 8 * ((lane >> 3) & 1), np * 2 + (lane >> 4))));
+            ldsm_x4_trans(b0, b1, b2, b3, vrow + (dh * 8 + np * 2 + (lane >> 4)) * 16);
             mma_f16_16816(o_acc[2 * np], pf[kk][0], pf[kk][1], pf[kk][2], pf[kk][3], b0, b1);
             mma_f16_16816(o_acc[2 * np + 1], pf[kk][0], pf[kk][1], pf[kk][2], pf[kk][3], b2, b3);
           }
         }
       }
-      __syncthreads();  // tile consumed
-      if (ti + 1 < n_tiles) {
-        store_tile();
-        __syncthreads();
+    };
+    for (int j = 0; j < n_chunks; ++j) {
+      stage_ready(j);
+      if (warp < 6) {
+        const unsigned char* kb = act + (j & 1) * kHalfBytes;
+        attend(kb, kb + kStageKeys * kRowStride, kRowStride, min(kStageKeys, n_cache - j * kStageKeys));
       }
+      __syncthreads();  // half j & 1 consumed
+      if (j + 2 < n_chunks) stage_issue(j + 2, kc, vc);
     }
+    if (warp < 6 && own_n > 0)
+      attend(reinterpret_cast<const unsigned char*>(ownk + static_cast<size_t>(own_lo) * kQS),
+             reinterpret_cast<const unsigned char*>(ownv + static_cast<size_t>(own_lo) * kQS), kQS * 2, own_n);
 
     // --- merge the 4 splits: stage this split's normalised partial (fp16) and
     // log-sum-exp locally, then send each row to the rank that owns it
-    __half* part = reinterpret_cast<__half*>(tile_k);  // [48][kD] (tile area, free now)
-    float* part_lse = reinterpret_cast<float*>(smem + L.rstd);
-    if (warp < 3) {
-      const int qr0 = warp * 16 + (lane >> 2);
+    __half* part = reinterpret_cast<__half*>(obuf);  // [48][kD] (tile area)
+    float* part_lse = reinterpret_cast<float*>(smem + L.lse);
+    if (warp < 6) {
+      const int qr0 = qt * 16 + (lane >> 2);
       const int qr1 = qr0 + 8;
       const float inv0 = l_run[0] > 0.f ? 1.f / l_run[0] : 0.f;
       const float inv1 = l_run[1] > 0.f ? 1.f / l_run[1] : 0.f;
 #pragma unroll
-      for (int n = 0; n < 16; ++n) {
-        const int c = n * 8 + 2 * (lane & 3);
+      for (int n = 0; n < 8; ++n) {
+        const int c = dh * 64 + n * 8 + 2 * (lane & 3);
         *reinterpret_cast<uint32_t*>(part + qr0 * kD + c) = pack_half2(o_acc[n][0] * inv0, o_acc[n][1] * inv0);
         *reinterpret_cast<uint32_t*>(part + qr1 * kD + c) = pack_half2(o_acc[n][2] * inv1, o_acc[n][3] * inv1);
       }
-      if ((lane & 3) == 0) {
+      if (dh == 0 && (lane & 3) == 0) {
         part_lse[qr0] = l_run[0] > 0.f ? m_run[0] + log2f(l_run[0]) : -CUDART_INF_F;
         part_lse[qr1] = l_run[1] > 0.f ? m_run[1] + log2f(l_run[1]) : -CUDART_INF_F;
       }
@@ -580,7 +691,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       st_cluster_f32(cluster_addr(recv_lse + rank * kRowsPerRank + tid - owner * kRowsPerRank, owner), part_lse[tid]);
     }
     cluster.sync();
-    // merged rows of o_h -> every partner's qbuf (now free) as the W_o input
+    // merged rows of o_h -> swizzled image in every partner's obuf (the W_o B operand)
     {
       const int r0 = rank * kRowsPerRank;
       for (int i = tid; i < kRowsPerRank * (kD / 4); i += kThr) {
@@ -609,79 +720,151 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         uint2 out;
         out.x = pack_half2(a0 * inv, a1 * inv);
         out.y = pack_half2(a2 * inv, a3 * inv);
-        *reinterpret_cast<uint2*>(qbuf + row * kQS + c) = out;
+        *reinterpret_cast<uint2*>(obuf + sw128_offset(kTokTile, row, c)) = out;
         if (p.attn_capture != nullptr && row < T)
           *reinterpret_cast<uint2*>(p.attn_capture + (static_cast<size_t>(layer) * T + row) * HD + head * kD + c) = out;
       }
     }
     __syncthreads();
-    push_rows(qbuf + rank * kRowsPerRank * kQS, kRowsPerRank, kQS * 2, kD * 2, rank, tid, kThr);
+    for (int i = tid; i < kRowsPerRank * (kD / 8) * (kCl - 1); i += kThr) {
+      const int peer_i = i / (kRowsPerRank * (kD / 8));
+      const int rest = i - peer_i * kRowsPerRank * (kD / 8);
+      const int row = rank * kRowsPerRank + rest / (kD / 8);
+      const int u = rest % (kD / 8);
+      const int peer = peer_i + (peer_i >= rank ? 1 : 0);
+      const uint32_t off = sw128_offset(kTokTile, row, u * 8);
+      st_cluster_v4(cluster_addr(obuf + off, peer), *reinterpret_cast<const uint4*>(obuf + off));
+    }
+    asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
     cluster.sync();  // o_h complete everywhere; ownk/ownv free for the transpose
 
-    // --- W_o: this CTA's 128 output columns for head h (8 blocks, one per warp)
-    {
-      const uint4* w = wait_chunk(q_chunk + (warp >> 2)) + (warp & 3) * (kD / 16) * 32;
-      float acc[6][4];
-      block_gemm(w, kD / 16, qbuf, kQS, acc, lane);
-      store_transposed(acc, warp * 16);
+    // --- W_o: this CTA's 128 output columns for head h, K = 128 (slots 0, 1)
+    if (warp == 0) {
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tc_fence_after();
+      for (int a = 0; a < 2; ++a) {
+        const bool ok = wait_chunk(q0 + kSlots + a);
+        if (ok && lane == 0) mma_slice(ring_a + a * kSlotBytes, smem_addr(obuf) + a * kActAtom, a == 0);
+        __syncwarp();
+      }
+      if (lane == 0) umma_commit(mma_bar);
+      __syncwarp();
     }
-    __syncthreads();
-    if (tid == 0)
-      for (int i = 0; i < 2; ++i) issue(q_chunk + i + kSlots);
-    q_chunk += 2;
+    wait_mma();
+    tmem_to_dstT();
+    if (tid == 0) {  // slots 0, 1 free (all of 0-5 for CTAs without phase B): next layer's QKV
+      const int n = in_b ? 2 : kSlots;
+      for (int i = 0; i < n; ++i) issue(q0 + kLayerChunks + i);
+    }
     scatter_add(Xm, Xc, rank * 128, head == 0);
     arrive(p.counters + sA + 1);
 
     // =========================== phase B ===========================
     if (in_b) {
       const int c = head;  // SwiGLU column block 64c..64c+63
-      wait_counter(p.counters + sA + 1, G, p.status);
+      wait_counter(p.counters + sA + 1, G, p.status, abort);
       {  // zero the buffer the next phase A accumulates into (this layer's input is consumed)
         const int e0 = static_cast<int>(static_cast<long long>(n_elem) * cta / n_b_ctas);
         const int e1 = static_cast<int>(static_cast<long long>(n_elem) * (cta + 1) / n_b_ctas);
         for (int e = e0 + tid; e < e1; e += kThr) __stcg(Xc + e, 0.f);
       }
       load_normalized(Xm);
-      __half* hsl = qbuf;  // [48][kHS] SwiGLU slice of this cluster
-      if (warp < 2) {     // 2 blocks: 8 gate + 8 up rows each -> 8 SwiGLU columns each
-        const uint4* w = wait_chunk(q_chunk + warp);
-        float acc[6][4];
-        block_gemm(w, d / 16, act, as, acc, lane);
-        const int col = rank * 16 + warp * 8 + (lane >> 2);
+      // gate/up: D[32 (+96 unused) rows x 48 tokens], 4 KB K slices in slots 2, 3
+      if (warp == 0) {
+        tc_fence_after();
+        for (int a = 0; a < d / 64; ++a) {
+          const int pos = kPersistAChunks + (a * kGuAtom) / kSlotBytes;
+          bool ok = true;
+          if ((a * kGuAtom) % kSlotBytes == 0) ok = wait_chunk(q0 + pos);
+          ok = ok && *abort == 0;
+          if (ok && lane == 0) mma_slice(ring_a + 2 * kSlotBytes + a * kGuAtom, act_a + a * kActAtom, a == 0);
+          __syncwarp();
+        }
+        if (lane == 0) umma_commit(mma_bar);
+        __syncwarp();
+      }
+      wait_mma();
+      // accumulator rows 0-15: gate of columns 16 rank + r, rows 16-31: the matching
+      // up rows. Warps 0 and 4 (the ones that reach TMEM lanes 0-31) copy them out
+      // as [32 rows][49] fp32; then every thread forms h = silu(gate) * up.
+      float* graw = dstT;
+      constexpr int kGS = kTokTile + 1;
+      if ((warp & 3) == 0) {
+        for (int c0 = warp == 0 ? 0 : 32; c0 < (warp == 0 ? 32 : 48); c0 += 16) {
+          float v[16];
+          __syncwarp();
+          tmem_ld16(tmem + static_cast<uint32_t>(c0), v);
 #pragma unroll
-        for (int t = 0; t < 6; ++t) {
-          const int m = t * 8 + 2 * (lane & 3);
-          const float h0 = acc[t][0] / (1.f + __expf(-acc[t][0])) * acc[t][2];
-          const float h1 = acc[t][1] / (1.f + __expf(-acc[t][1])) * acc[t][3];
-          hsl[m * kHS + col] = __float2half_rn(h0);
-          hsl[(m + 1) * kHS + col] = __float2half_rn(h1);
+          for (int j = 0; j < 16; ++j) graw[lane * kGS + c0 + j] = v[j];
         }
       }
       __syncthreads();
-      if (tid == 0)
-        for (int i = 0; i < 2; ++i) issue(q_chunk + i + kSlots);
-      q_chunk += 2;
-      push_rows(hsl + rank * 16, kTokTile, kHS * 2, 32, rank, tid, kThr);
-      cluster.sync();  // SwiGLU slice complete everywhere
-      {
-        const uint4* w = wait_chunk(q_chunk) + warp * (64 / 16) * 32;
-        float acc[6][4];
-        block_gemm(w, 64 / 16, hsl, kHS, acc, lane);
-        store_transposed(acc, warp * 16);
+      for (int i = tid; i < kTokTile * 16; i += kThr) {
+        const int t = i >> 4;
+        const int cc = i & 15;
+        const float g = graw[cc * kGS + t];
+        const float u = graw[(16 + cc) * kGS + t];
+        *reinterpret_cast<__half*>(hsl + sw128_offset(kTokTile, t, rank * 16 + cc)) =
+            __float2half_rn(__fdividef(g, 1.f + __expf(-g)) * u);
       }
+      tc_fence_before();
       __syncthreads();
-      if (tid == 0) issue(q_chunk + kSlots);
-      q_chunk += 1;
+      if (tid == 0)  // slots 2, 3 free: next layer's QKV
+        for (int i = 2; i < 4; ++i) issue(q0 + kLayerChunks + i);
+      // this rank's 16 columns (two 16-byte units per token row) to the partners
+      for (int i = tid; i < kTokTile * 2 * (kCl - 1); i += kThr) {
+        const int peer_i = i / (kTokTile * 2);
+        const int rest = i - peer_i * kTokTile * 2;
+        const int t = rest >> 1;
+        const int u = rank * 2 + (rest & 1);
+        const int peer = peer_i + (peer_i >= rank ? 1 : 0);
+        const uint32_t off = sw128_offset(kTokTile, t, u * 8);
+        st_cluster_v4(cluster_addr(hsl + off, peer), *reinterpret_cast<const uint4*>(hsl + off));
+      }
+      asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+      cluster.sync();  // SwiGLU slice complete everywhere
+      // --- W_d: 128 output columns over the cluster's 64 SwiGLU inputs (slot 4)
+      if (warp == 0) {
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        tc_fence_after();
+        const bool ok = wait_chunk(q0 + kPersistAChunks + 2);
+        if (ok && lane == 0) mma_slice(ring_a + 4 * kSlotBytes, smem_addr(hsl), true);
+        __syncwarp();
+        if (lane == 0) umma_commit(mma_bar);
+        __syncwarp();
+      }
+      wait_mma();
+      tmem_to_dstT();
+      if (tid == 0)  // slots 4, 5 free: next layer's QKV
+        for (int i = 4; i < kSlots; ++i) issue(q0 + kLayerChunks + i);
       float* Xn = X0 + static_cast<size_t>((sA + 2) % 3) * xs;
       scatter_add(Xn, Xm, rank * 128, c == 0);
       arrive(p.counters + sA + 2);
-      (void)c;
     }
   }
 
+  // a tick that timed out may have skipped waits: let this CTA's last copies land
+  // (bounded) before the shared memory is released
+  if (tid == 0 && *abort)
+    for (int q = total_chunks - kSlots; q < total_chunks; ++q)
+      if (q >= 0 && !is_empty(q)) {
+        const unsigned long long t0 = global_timer_ns();
+        uint32_t done = 0;
+        while (!done && global_timer_ns() - t0 < 100000000ull)
+          asm volatile(
+              "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+              : "=r"(done)
+              : "r"(smem_addr(full + q % kSlots)), "r"(static_cast<uint32_t>((q / kSlots) & 1))
+              : "memory");
+      }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+
   // =========================== head ===========================
   if (cta == 0) {
-    wait_counter(p.counters + 2 * p.n_layers, n_b_ctas, p.status);
+    wait_counter(p.counters + 2 * p.n_layers, n_b_ctas, p.status, abort);
     const float* Xf = X0 + static_cast<size_t>((2 * p.n_layers) % 3) * xs;
     for (int j = warp; j < p.n_waypoints; j += kThr / 32) {
       const float* xr = Xf + static_cast<size_t>(j) * d;
