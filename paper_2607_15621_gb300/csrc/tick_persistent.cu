@@ -484,14 +484,13 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     const CT* kc = static_cast<const CT*>(p.targs->k_cache[layer]);
     const CT* vc = static_cast<const CT*>(p.targs->v_cache[layer]);
 
-    // L2 prefetch of this CTA's cache rows of this layer
-    if (warp == 0) {
-      const long long c_end = min(kend, Lc);
-      for (long long key = kbeg + lane; key < c_end; key += 32) {
-        const size_t row = (static_cast<size_t>(o_lo + key) * p.H + head) * kD;
-        prefetch_l2(kc + row, kD * sizeof(CT));
-        prefetch_l2(vc + row, kD * sizeof(CT));
-      }
+    // L2 prefetch of this layer's cache: CTA c takes whole token rows (all heads,
+    // contiguous) t = c, c + G, ..., spread over its threads, so the grid issues a
+    // handful of large prefetches instead of one per (token, head) row
+    for (long long t = cta + static_cast<long long>(G) * tid; t < Lc; t += static_cast<long long>(G) * kThr) {
+      const size_t row = static_cast<size_t>(o_lo + t) * p.H * kD;
+      prefetch_l2(kc + row, static_cast<uint32_t>(p.H * kD * sizeof(CT)));
+      prefetch_l2(vc + row, static_cast<uint32_t>(p.H * kD * sizeof(CT)));
     }
 
     // =========================== phase A ===========================
