@@ -5,7 +5,7 @@
 //
 // Split-KV flash decoding: the L_b + T keys of a vehicle are cut into
 // n_splits near-equal ranges; one CTA (3 warps x 16 queries = 48 query rows)
-// streams its range in 64-key chunks. Chunks are staged raw (bf16 / fp32 cache
+// streams its range in 32-key chunks. Chunks are staged raw (bf16 / fp32 cache
 // rows, fp16 own rows) with 16-byte cp.async into a double buffer, converted
 // once to fp16 into an XOR-swizzled tile, and consumed by mma.sync m16n8k16
 // (S = Q K^T, then O += P V with P kept in registers) under an online softmax
@@ -31,7 +31,19 @@ namespace {
 constexpr int kMaxClusterSplits = 8;
 constexpr int kWarps = 3;
 constexpr int kThreads = kWarps * 32;
-constexpr int kChunk = 64;
+#ifndef FSX_ATTN_CHUNK
+#define FSX_ATTN_CHUNK 32
+#endif
+#ifndef FSX_ATTN_MIN_CTAS
+#define FSX_ATTN_MIN_CTAS 3
+#endif
+#ifndef FSX_ATTN_RAW_STAGES
+#define FSX_ATTN_RAW_STAGES 2
+#endif
+constexpr int kChunk = FSX_ATTN_CHUNK;  // keys per staged chunk
+constexpr int kRawStages = FSX_ATTN_RAW_STAGES;  // raw chunks staged (in flight while one is computed)
+constexpr int kNT = kChunk / 8;         // 8-key n tiles of S
+constexpr int kKS = kChunk / 16;        // 16-key k steps of P V
 constexpr int kD = kHeadDim;           // 128
 constexpr int kUnits = kD * 2 / 16;    // 16-byte units per fp16 row (16)
 
@@ -40,13 +52,21 @@ struct CacheRow {
   static constexpr int kBytes = kD * static_cast<int>(sizeof(CT));
 };
 
-// raw staging: [2 stages][K|V][kChunk rows][row bytes]; compute tiles: fp16 [K|V][kChunk][kD] swizzled
+// raw staging: [kRawStages][K|V][kChunk rows][row bytes]; compute tiles: fp16 [K|V][kChunk][kD] swizzled
 template <typename CT>
 __host__ __device__ constexpr size_t attn_smem_bytes() {
-  return static_cast<size_t>(2) * 2 * kChunk * CacheRow<CT>::kBytes + static_cast<size_t>(2) * kChunk * kD * 2;
+  return static_cast<size_t>(kRawStages) * 2 * kChunk * CacheRow<CT>::kBytes + static_cast<size_t>(2) * kChunk * kD * 2;
 }
 
 __device__ __forceinline__ int swz(int row, int unit) { return row * kUnits + (unit ^ (row & 7)); }
+
+// wait until at most n of this thread's cp.async groups are pending
+__device__ __forceinline__ void cp_async_wait_n(int n) {
+  if (n <= 0) cp_async_wait<0>();
+  else if (n == 1) cp_async_wait<1>();
+  else if (n == 2) cp_async_wait<2>();
+  else cp_async_wait<3>();
+}
 
 template <typename CT>
 __device__ __forceinline__ void convert_unit(const unsigned char* raw, uint4* dst, bool own);
@@ -74,12 +94,15 @@ __device__ __forceinline__ void convert_unit<float>(const unsigned char* raw, ui
   }
 }
 
+static_assert((kTokTile + kMaxClusterSplits - 1) * (kD + 1) * 4 <= (2 * kRawStages + 2) * kChunk * kD * 2,
+              "the cluster merge buffers must fit in the staging memory");
+
 template <typename CT, bool CM>
-__global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p) {
+__global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kernel(const AttnArgs p) {
   extern __shared__ __align__(128) unsigned char smem[];
   constexpr int RB = CacheRow<CT>::kBytes;
-  unsigned char* raw = smem;                                              // [2][2][kChunk][RB]
-  uint4* tile = reinterpret_cast<uint4*>(smem + static_cast<size_t>(2) * 2 * kChunk * RB);
+  unsigned char* raw = smem;                                              // [kRawStages][2][kChunk][RB]
+  uint4* tile = reinterpret_cast<uint4*>(smem + static_cast<size_t>(kRawStages) * 2 * kChunk * RB);
   uint4* kt = tile;                      // fp16 K chunk, swizzled
   uint4* vt = tile + kChunk * kUnits;    // fp16 V chunk, swizzled
 
@@ -200,12 +223,11 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
   const float scale_log2 = 1.4426950408889634f * rsqrtf(static_cast<float>(kD));
 
   const int n_chunks = empty_range ? 0 : static_cast<int>((kend - kbeg + kChunk - 1) / kChunk);
-  if (n_chunks > 0) issue_chunk(0, 0);
-  if (n_chunks > 1) issue_chunk(1, 1);
+  for (int i = 0; i < kRawStages && i < n_chunks; ++i) issue_chunk(i, i);
 
   for (int c = 0; c < n_chunks; ++c) {
-    const int s = c & 1;
-    if (c + 1 < n_chunks) cp_async_wait<1>(); else cp_async_wait<0>();
+    const int s = c % kRawStages;
+    cp_async_wait_n(min(kRawStages - 1, n_chunks - 1 - c));  // chunk c landed
     __syncthreads();  // raw stage s complete for everyone; previous tile consumers done
 
     // ---- convert raw stage s -> fp16 swizzled tiles (rows beyond the range are zero)
@@ -232,12 +254,12 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
       }
     }
     __syncthreads();  // tiles ready, raw stage s free
-    if (c + 2 < n_chunks) issue_chunk(c + 2, s);
+    if (c + kRawStages < n_chunks) issue_chunk(c + kRawStages, s);
 
-    // ---- S = Q K^T for 16 queries x 64 keys
-    float sc[8][4];
+    // ---- S = Q K^T for 16 queries x kChunk keys
+    float sc[kNT][4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < kNT; ++j) {
 #pragma unroll
       for (int e = 0; e < 4; ++e) sc[j][e] = 0.f;
 #pragma unroll
@@ -253,7 +275,7 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
     // ---- online softmax (log2 domain), masking keys past the range
     float mx[2] = {-CUDART_INF_F, -CUDART_INF_F};
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < kNT; ++j) {
       const int key = j * 8 + 2 * (lane & 3);
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
@@ -275,9 +297,9 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
       alpha[r] = exp2f(m_run[r] - m_new[r]);
       m_run[r] = m_new[r];
     }
-    uint32_t pf[4][4];  // P as A fragments, 4 k16 steps of 16 keys
+    uint32_t pf[kKS][4];  // P as A fragments, one per k16 step of 16 keys
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < kNT; ++j) {
       const float p0 = exp2f(sc[j][0] - m_new[0]);
       const float p1 = exp2f(sc[j][1] - m_new[0]);
       const float p2 = exp2f(sc[j][2] - m_new[1]);
@@ -308,7 +330,7 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
     }
     // ---- O += P V
 #pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
+    for (int kk = 0; kk < kKS; ++kk) {
 #pragma unroll
       for (int np = 0; np < 8; ++np) {  // pairs of 8-wide d tiles
         const int row = kk * 16 + (lane & 7) + 8 * ((lane >> 3) & 1);
@@ -333,7 +355,9 @@ __global__ void __launch_bounds__(kThreads) attn_splitkv_kernel(const AttnArgs p
     const int S = static_cast<int>(cluster.num_blocks());
     const int rank = static_cast<int>(cluster.block_rank());
     const int rows_per = (kTokTile + S - 1) / S;
-    float* rPo = reinterpret_cast<float*>(tile);            // [S][rows_per][kD]
+    // [S][rows_per][kD] + [S][rows_per]: at most 55 rows (S <= 8), 28.4 KB, placed
+    // at the start of the (idle) staging memory (48 KB or more; checked above)
+    float* rPo = reinterpret_cast<float*>(smem);
     float* rLse = rPo + static_cast<size_t>(S) * rows_per * kD;  // [S][rows_per]
     cluster.sync();  // every split is done with its tiles
     {
