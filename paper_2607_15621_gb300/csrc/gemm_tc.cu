@@ -3,20 +3,23 @@
 // token count M = 42 B makes them real dense contractions.
 //
 // D[128 weight rows, BN tokens] = W_tile[128, K] . A[BN tokens, K]^T, fp16
-// operands, fp32 accumulation in tensor memory. Each CTA owns one 128-row
-// weight tile and one BN-token block and walks K in 64-wide steps through a
-// 4-stage shared-memory pipeline:
-//   warp 0 (one lane): producer -- the weight tile arrives as one 16 KB bulk
-//     copy of a pre-swizzled image (packed at fsx_create in the 128-byte
-//     swizzle layout the MMA reads), the token tile by a 2-D TMA load with the
-//     same swizzle (rows past M read as zeros);
-//   warp 1 (one lane): issues tcgen05.mma (M=128, N=BN, K=16) x4 per stage and
-//     commits each stage back to the producer;
-//   all 4 warps: epilogue -- tcgen05.ld of their 32 TMEM lanes (weight rows)
-//     into a token-major tile in the idle pipeline buffers, then 16-byte
-//     stores: fp16 output, SwiGLU (gate rows 16j..16j+7 next to their up rows),
-//     or the fp32 residual update (each element owned by one thread), which
-//     also emits each token's sum of x^2 over its 128 columns.
+// operands, fp32 accumulation in tensor memory. The kernel is persistent: one
+// CTA per SM walks the (weight tile, token block) tiles gridDim.x apart, and
+// its warps specialise:
+//   warp 0 (one lane): producer -- per 64-wide K step, the weight tile arrives
+//     as one 16 KB bulk copy of a pre-swizzled image (packed at fsx_create in
+//     the 128-byte swizzle layout the MMA reads), the token tile by a 2-D TMA
+//     load with the same swizzle (rows past M read as zeros), through a
+//     4-stage ring that runs on across tile boundaries;
+//   warp 1 (one lane): issues tcgen05.mma (M=128, N=BN, K=16) x4 per stage,
+//     releases each stage to the producer, and alternates between two
+//     accumulators in tensor memory, so the MMAs of tile i+1 run while the
+//     epilogue drains tile i;
+//   warps 2-5: epilogue -- tcgen05.ld of their 32 TMEM lanes (weight rows) in
+//     chunks of tokens into a token-major staging tile, then 16-byte stores:
+//     fp16 output, SwiGLU (gate rows 16j..16j+7 next to their up rows), or the
+//     fp32 residual update (each element owned by one thread), which also
+//     emits each token's sum of x^2 over its 128 columns.
 // RMSNorm-fused GEMMs (QKV, gate/up) take the fp16 copy of the residual stream
 // as A, with the norm gain folded into the packed weights, and scale each
 // token's result by 1/rms built from those per-128-column sums in a fixed
@@ -31,11 +34,16 @@ namespace fsx {
 
 namespace {
 
-constexpr int kTcThreads = 128;
+constexpr int kEpiGroups = 3;         // epilogue groups of 4 warps (one per TMEM lane quadrant)
+constexpr int kEpiThreads = kEpiGroups * 128;
+constexpr int kTcThreads = 64 + kEpiThreads;  // producer warp, MMA warp, epilogue groups
 constexpr int kStages = 4;
-constexpr int kTileN = 128;           // weight rows per CTA (MMA M)
+constexpr int kTileN = 128;           // weight rows per tile (MMA M)
 constexpr int kTileK = 64;            // K per stage (128 bytes of fp16: one swizzle span)
 constexpr int kWTileBytes = kTileN * kTileK * 2;  // 16 KB
+constexpr int kEpiChunk = 32;                     // tokens per epilogue round of one half
+constexpr int kStgHalfBytes = 9216;               // fp16 staging of one group: 32 tokens x (128 + 8) halves
+constexpr int kSspBytes = ((kEpiGroups * 32 * 4 * 4 + 1023) / 1024) * 1024;  // x^2 partials [groups][32][4]
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
   asm volatile(
@@ -45,15 +53,34 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       : "memory");
 }
 
+// barrier among the 4 warps of epilogue group h (ids 1 .. kEpiGroups) / all epilogue warps
+__device__ __forceinline__ void half_sync(int h) { asm volatile("bar.sync %0, 128;" ::"r"(1 + h) : "memory"); }
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync %0, %1;" ::"n"(1 + kEpiGroups), "n"(kEpiThreads) : "memory"); }
+
 template <int BN>
 __host__ __device__ constexpr int tc_stage_bytes() {
   return kWTileBytes + BN * kTileK * 2;
 }
 
 template <int BN>
+__host__ __device__ constexpr int tc_rstd_bytes() {  // 1/rms of the tokens, double-buffered by tile parity
+  return ((2 * BN * 4 + 1023) / 1024) * 1024;
+}
+// a 32-token chunk read of the 1/rms buffer may run past BN (last chunk of BN = 48)
+static_assert(tc_rstd_bytes<48>() >= (2 * 48 + 32) * 4, "1/rms buffer too small for a 32-token read");
+static_assert(kStgHalfBytes % 1024 == 0 && kSspBytes % 1024 == 0, "the stage ring must stay 1024-byte aligned");
+
+template <int BN>
 __host__ __device__ constexpr int tc_smem_bytes() {
-  return 1024 /* barriers, tmem address */ + ((BN * 4 + 1023) / 1024) * 1024 /* 1/rms */ + 1024 /* alignment slack */ +
-         kStages * tc_stage_bytes<BN>();
+  return 1024 /* barriers, tmem address */ + tc_rstd_bytes<BN>() + kSspBytes + kEpiGroups * kStgHalfBytes +
+         1024 /* alignment slack */ + kStages * tc_stage_bytes<BN>();
+}
+
+static_assert(tc_smem_bytes<256>() <= 232448, "shared memory of the widest tile exceeds the per-block limit");
+
+template <int BN>
+__host__ __device__ constexpr uint32_t tc_tmem_cols() {  // two accumulators, power of two >= 32
+  return 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512)));
 }
 
 template <int BN, int EPI, bool NORM>
@@ -65,179 +92,266 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(base);
   uint64_t* empty = full + kStages;
-  uint64_t* done = empty + kStages;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
-  float* s_rstd = reinterpret_cast<float*>(base + 1024);
-  unsigned char* stages = base + 1024 + ((BN * 4 + 1023) / 1024) * 1024;  // after the 1/rms block
+  uint64_t* tmem_full = empty + kStages;   // [2] accumulator ready for the epilogue
+  uint64_t* tmem_empty = tmem_full + 2;    // [2] accumulator drained
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tmem_empty + 2);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);  // a wait of this CTA timed out
+  float* s_rstd = reinterpret_cast<float*>(base + 1024);                    // [2][BN]
+  float* s_ssp = reinterpret_cast<float*>(base + 1024 + tc_rstd_bytes<BN>());  // [groups][32 tokens][4 quadrants]
+  unsigned char* stg = base + 1024 + tc_rstd_bytes<BN>() + kSspBytes;        // [groups] fp16 staging
+  unsigned char* stages = stg + kEpiGroups * kStgHalfBytes;
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const int lane = tid & 31;
-  const int n0 = blockIdx.x * kTileN;  // first weight row
-  const int m0 = blockIdx.y * BN;      // first token
   const int KT = p.K / kTileK;
+  const int tiles_n = p.N / kTileN;
+  const int n_tiles = tiles_n * ((p.M + BN - 1) / BN);
   constexpr int kAbytes = BN * kTileK * 2;
-  constexpr uint32_t kTmemCols = BN <= 32 ? 32 : (BN <= 64 ? 64 : (BN <= 128 ? 128 : 256));
+  constexpr uint32_t kTmemCols = tc_tmem_cols<BN>();
+  // bounded wait that gives up at once after an earlier timeout of this CTA
+  auto wait = [&](uint64_t* bar, uint32_t parity) {
+    if (*abort) return;
+    if (!mbar_wait(bar, parity, p.status)) *abort = 1;
+  };
 
   pdl_launch_dependents();
   if (tid == 0) {
+    *abort = 0;
     for (int s = 0; s < kStages; ++s) {
       mbar_init(full + s, 1);
       mbar_init(empty + s, 1);
     }
-    mbar_init(done, 1);
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tmem_full + a, 1);
+      mbar_init(tmem_empty + a, 4 * kEpiGroups);  // one arrival per epilogue warp
+    }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
-  if (warp == 0) {  // tensor memory for the accumulator: BN fp32 columns x 128 lanes
+  if (warp == 0) {  // tensor memory for two accumulators of BN fp32 columns x 128 lanes
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(tmem_slot)),
                  "r"(kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  tc_fence_before();
   __syncthreads();
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  tc_fence_after();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(tmem_slot);
 
   if (warp == 0) {
-    // ---- producer warp (converged; lane 0 issues): weights may stream before
-    // the previous kernel finished, the token tiles only after it
-    const unsigned char* wtile = p.w + static_cast<size_t>(blockIdx.x) * KT * kWTileBytes;
-    const int pre = KT < kStages ? KT : kStages;
-    if (lane == 0) {
-      for (int kt = 0; kt < pre; ++kt) {
-        mbar_arrive_expect_tx(full + kt, kWTileBytes + kAbytes);
-        bulk_g2s(stages + kt * tc_stage_bytes<BN>(), wtile + static_cast<size_t>(kt) * kWTileBytes, kWTileBytes,
-                 full + kt);
+    // ---- producer (converged; lane 0 issues). Stage g of this CTA's stream is
+    // K step g % KT of its tile g / KT. Weights may stream before the previous
+    // kernel finished, the token tiles only after it.
+    const int my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - static_cast<int>(blockIdx.x)) / static_cast<int>(gridDim.x) + 1 : 0;
+    const int total = my_tiles * KT;
+    auto w_src = [&](int g) {
+      const int t = static_cast<int>(blockIdx.x) + (g / KT) * static_cast<int>(gridDim.x);
+      return p.w + (static_cast<size_t>(t % tiles_n) * KT + g % KT) * kWTileBytes;
+    };
+    const int pre = total < kStages ? total : kStages;
+    if (lane == 0)
+      for (int g = 0; g < pre; ++g) {
+        mbar_arrive_expect_tx(full + g, kWTileBytes + kAbytes);
+        bulk_g2s(stages + g * tc_stage_bytes<BN>(), w_src(g), kWTileBytes, full + g);
       }
-    }
     __syncwarp();
     pdl_wait();
-    for (int kt = 0; kt < KT; ++kt) {
-      const int s = kt % kStages;
+    for (int g = 0; g < total; ++g) {
+      const int s = g % kStages;
       unsigned char* st = stages + s * tc_stage_bytes<BN>();
-      if (kt >= kStages) mbar_wait(empty + s, static_cast<uint32_t>(((kt / kStages) - 1) & 1), p.status);
+      if (g >= kStages) wait(empty + s, static_cast<uint32_t>(((g / kStages) - 1) & 1));
       if (lane == 0) {
-        if (kt >= kStages) {
+        const int t = static_cast<int>(blockIdx.x) + (g / KT) * static_cast<int>(gridDim.x);
+        if (g >= kStages) {
           mbar_arrive_expect_tx(full + s, kWTileBytes + kAbytes);
-          bulk_g2s(st, wtile + static_cast<size_t>(kt) * kWTileBytes, kWTileBytes, full + s);
+          bulk_g2s(st, w_src(g), kWTileBytes, full + s);
         }
-        tma_load_2d(st + kWTileBytes, &map_a, kt * kTileK, m0, full + s);
+        tma_load_2d(st + kWTileBytes, &map_a, (g % KT) * kTileK, (t / tiles_n) * BN, full + s);
       }
       __syncwarp();
     }
+    // after a timeout the MMA warp may have skipped its waits: let the copies still in
+    // flight land (bounded) before the shared memory is released
+    if (*abort && lane == 0)
+      for (int g = total - kStages; g < total; ++g) {
+        if (g < 0) continue;
+        const unsigned long long t0 = global_timer_ns();
+        uint32_t done = 0;
+        while (!done && global_timer_ns() - t0 < 100000000ull)
+          asm volatile(
+              "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+              : "=r"(done)
+              : "r"(smem_addr(full + g % kStages)), "r"(static_cast<uint32_t>((g / kStages) & 1))
+              : "memory");
+      }
+    __syncwarp();
   } else if (warp == 1) {
-    // ---- MMA warp (converged; lane 0 issues)
+    // ---- MMA issuer (converged; lane 0 issues)
     pdl_wait();
     constexpr uint32_t idesc = idesc_f16(kTileN, BN);
-    for (int kt = 0; kt < KT; ++kt) {
-      const int s = kt % kStages;
-      mbar_wait(full + s, static_cast<uint32_t>((kt / kStages) & 1), p.status);
-      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      if (lane == 0) {
-        const uint32_t a_base = smem_addr(stages + s * tc_stage_bytes<BN>());
-        const uint32_t b_base = a_base + kWTileBytes;
+    int g = 0;
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+      const int acc = i & 1;
+      if (i >= 2) wait(tmem_empty + acc, static_cast<uint32_t>(((i >> 1) - 1) & 1));
+      tc_fence_after();
+      const uint32_t d = tmem + static_cast<uint32_t>(acc * BN);
+      for (int kt = 0; kt < KT; ++kt, ++g) {
+        const int s = g % kStages;
+        wait(full + s, static_cast<uint32_t>((g / kStages) & 1));
+        tc_fence_after();
+        if (lane == 0) {
+          const uint32_t a_base = smem_addr(stages + s * tc_stage_bytes<BN>());
+          const uint32_t b_base = a_base + kWTileBytes;
 #pragma unroll
-        for (int k = 0; k < kTileK / 16; ++k)
-          umma_f16(tmem, sw128_desc(a_base + k * 32), sw128_desc(b_base + k * 32), idesc, (kt > 0 || k > 0) ? 1u : 0u);
-        umma_commit(empty + s);
+          for (int k = 0; k < kTileK / 16; ++k)
+            umma_f16(d, sw128_desc(a_base + k * 32), sw128_desc(b_base + k * 32), idesc, (kt > 0 || k > 0) ? 1u : 0u);
+          umma_commit(empty + s);
+        }
+        __syncwarp();
       }
+      if (lane == 0) umma_commit(tmem_full + acc);
       __syncwarp();
     }
-    if (lane == 0) umma_commit(done);
-    __syncwarp();
-  }
-
-  // ---- epilogue: every warp reads its 32 lanes (weight rows n0 + 32 warp + lane)
-  pdl_wait();  // the residual stream written by the previous kernel is read below
-  if (NORM) {  // 1/rms of the tile's tokens from the per-128-column partial sums of x^2
-    for (int t = tid; t < BN; t += kTcThreads) {
-      float ss = 0.f;
-      if (m0 + t < p.M)
-        for (int j = 0; j < p.n_ss; ++j) ss += __ldcg(p.ss_in + static_cast<size_t>(j) * p.ss_stride + m0 + t);
-      s_rstd[t] = rsqrtf(ss / static_cast<float>(p.K) + 1e-6f);
-    }
-  }
-  mbar_wait(done, 0, p.status);
-  __syncthreads();  // 1/rms visible
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-  const int row = warp * 32 + lane;
-  const uint32_t taddr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-  // TMEM -> registers -> token-major tile in the (now idle) pipeline buffers
-  constexpr int kSH = kTileN + 8;  // fp16 row stride (store)
-  constexpr int kSG = 64 + 8;      // fp16 row stride (SwiGLU: 64 columns per tile)
-  constexpr int kSF = kTileN + 4;  // fp32 row stride (residual)
-  __half* tH = reinterpret_cast<__half*>(stages);
-  float* tF = reinterpret_cast<float*>(stages);
-  for (int c0 = 0; c0 < BN; c0 += 16) {
-    float v[16];
-    __syncwarp();  // tcgen05.ld.sync.aligned needs the whole warp converged
-    tmem_ld16(taddr + static_cast<uint32_t>(c0), v);
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      float val = v[j];
-      if (NORM) val *= s_rstd[c0 + j];
-      if (EPI == kEpiStore) {
-        tH[(c0 + j) * kSH + row] = __float2half_rn(val);
-      } else if (EPI == kEpiResidual) {
-        tF[(c0 + j) * kSF + row] = val;
-      } else {  // SwiGLU: lane l (l % 16 < 8) holds a gate row, lane l + 8 its up row
-        const float up = __shfl_down_sync(0xffffffffu, val, 8);
-        const __half hv = __float2half_rn(__fdividef(val, 1.f + __expf(-val)) * up);
-        if ((lane & 8) == 0) tH[(c0 + j) * kSG + (row >> 4) * 8 + (lane & 7)] = hv;
-      }
-    }
-  }
-  __syncthreads();
-  // coalesced 16-byte stores of the tile's token rows
-  if (EPI == kEpiStore) {
-    for (int i = tid; i < BN * (kTileN / 8); i += kTcThreads) {
-      const int t = i / (kTileN / 8);
-      const int u = i % (kTileN / 8);
-      if (m0 + t < p.M)
-        *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m0 + t) * p.ldy + n0 + u * 8) =
-            *reinterpret_cast<const uint4*>(tH + t * kSH + u * 8);
-    }
-  } else if (EPI == kEpiSwiglu) {
-    for (int i = tid; i < BN * 8; i += kTcThreads) {
-      const int t = i >> 3;
-      const int u = i & 7;
-      if (m0 + t < p.M)
-        *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m0 + t) * p.ldy + n0 / 2 + u * 8) =
-            *reinterpret_cast<const uint4*>(tH + t * kSG + u * 8);
-    }
   } else {
-    // warp w handles token rows w, w+4, ...: lane = 4-column group, so a warp covers
-    // one full 128-column row and reduces its x^2 partial with shuffles
-    constexpr int kRows = BN / 4;
-    constexpr int kBatch = kRows % 8 == 0 ? 8 : 4;  // divides kRows (12, 32 or 64)
-    for (int r0 = 0; r0 < kRows; r0 += kBatch) {
-      float4 a[kBatch];
-#pragma unroll
-      for (int b = 0; b < kBatch; ++b) {
-        const int t = (r0 + b) * 4 + warp;
-        a[b] = m0 + t < p.M ? *reinterpret_cast<const float4*>(p.xo + static_cast<size_t>(m0 + t) * p.ldxo + n0 + lane * 4)
-                            : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-#pragma unroll
-      for (int b = 0; b < kBatch; ++b) {
-        const int t = (r0 + b) * 4 + warp;
-        const float4 r = *reinterpret_cast<const float4*>(tF + t * kSF + lane * 4);
-        const float4 x = make_float4(a[b].x + r.x, a[b].y + r.y, a[b].z + r.z, a[b].w + r.w);
-        const float ss = warp_sum(x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w);
-        if (m0 + t < p.M) {
-          const size_t idx = static_cast<size_t>(m0 + t) * p.ldxo + n0 + lane * 4;
-          *reinterpret_cast<float4*>(p.xo + idx) = x;
-          uint2 pk;
-          pk.x = pack_half2(x.x, x.y);
-          pk.y = pack_half2(x.z, x.w);
-          *reinterpret_cast<uint2*>(p.xo16 + idx) = pk;
-          if (lane == 0 && p.ss_out != nullptr) p.ss_out[static_cast<size_t>(blockIdx.x) * p.ss_stride + m0 + t] = ss;
+    // ---- epilogue: groups of 4 warps (warps 2-5, 6-9, ...) take the 32-token chunks
+    // of a tile in turn; in each group TMEM lane quadrant q = warp % 4 holds weight
+    // rows 32q..32q+31 (this thread: row 32q + lane)
+    pdl_wait();  // the residual stream written by the previous kernel is read below
+    const int etid = tid - 64;
+    const int half = etid >> 7;  // epilogue group
+    const int htid = etid & 127;
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    constexpr int kSH = kTileN + 8;  // fp16 row stride (store)
+    constexpr int kSG = 64 + 8;      // fp16 row stride (SwiGLU: 64 columns per tile)
+    __half* tH = reinterpret_cast<__half*>(stg + half * kStgHalfBytes);
+    float* ssp = s_ssp + half * kEpiChunk * 4;
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+      const int acc = i & 1;
+      const int n0 = (t % tiles_n) * kTileN;
+      const int m0 = (t / tiles_n) * BN;
+      float* rstd = s_rstd + acc * BN;
+      if (NORM) {  // 1/rms of the tile's tokens from the per-128-column partial sums of x^2
+        for (int tt = etid; tt < BN; tt += kEpiThreads) {
+          float ss = 0.f;
+          if (m0 + tt < p.M)
+            for (int j = 0; j < p.n_ss; ++j) ss += __ldcg(p.ss_in + static_cast<size_t>(j) * p.ss_stride + m0 + tt);
+          rstd[tt] = rsqrtf(ss / static_cast<float>(p.K) + 1e-6f);
         }
       }
+      wait(tmem_full + acc, static_cast<uint32_t>((i >> 1) & 1));
+      tc_fence_after();
+      epi_sync();  // 1/rms visible to both halves; both halves are past the previous tile
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      for (int c0 = half * kEpiChunk; c0 < BN; c0 += kEpiGroups * kEpiChunk) {
+        const int nc = BN - c0 < kEpiChunk ? BN - c0 : kEpiChunk;  // 16 for the last chunk of BN = 48
+        uint32_t r[32];
+        __syncwarp();  // tcgen05.ld.sync.aligned needs the whole warp converged
+        if (nc == kEpiChunk) {
+          tmem_ld32_issue(taddr + static_cast<uint32_t>(c0), r);
+          tmem_wait_ld32(r);
+        } else {
+          float v16[16];
+          tmem_ld16(taddr + static_cast<uint32_t>(c0), v16);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) r[j] = __float_as_uint(v16[j]);
+#pragma unroll
+          for (int j = 16; j < 32; ++j) r[j] = 0u;
+        }
+        if (EPI == kEpiResidual) {
+          // x[m, n0 + row] += D[row, m]: lanes hold consecutive columns, so every access
+          // of the warp is one contiguous 128-byte row piece
+          const int n_ok = min(nc, p.M - (m0 + c0));  // valid tokens of the chunk
+          float* px = p.xo + static_cast<size_t>(m0 + c0) * p.ldxo + n0 + row;
+          __half* ph = p.xo16 + static_cast<size_t>(m0 + c0) * p.ldxo + n0 + row;
+          float x[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j)  // every load in flight before the first store
+            x[j] = j < n_ok ? __ldcg(px + static_cast<size_t>(j) * p.ldxo) : 0.f;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            x[j] += __uint_as_float(r[j]);
+            if (j < n_ok) {
+              px[static_cast<size_t>(j) * p.ldxo] = x[j];
+              ph[static_cast<size_t>(j) * p.ldxo] = __float2half_rn(x[j]);
+            }
+            x[j] = j < n_ok ? x[j] * x[j] : 0.f;
+          }
+          // 32 tokens x 32 lanes of x^2 -> lane l holds this quadrant's sum for token l
+#pragma unroll
+          for (int sh = 16; sh > 0; sh >>= 1) {
+            const bool upper = (lane & sh) != 0;
+#pragma unroll
+            for (int j = 0; j < sh; ++j) {
+              const float send = upper ? x[j] : x[j + sh];
+              const float keep = upper ? x[j + sh] : x[j];
+              x[j] = keep + __shfl_xor_sync(0xffffffffu, send, sh);
+            }
+          }
+          ssp[lane * 4 + q] = x[0];
+          half_sync(half);
+          if (htid < nc && p.ss_out != nullptr && m0 + c0 + htid < p.M)  // fixed quadrant order
+            p.ss_out[static_cast<size_t>(t % tiles_n) * p.ss_stride + m0 + c0 + htid] =
+                ((ssp[htid * 4 + 0] + ssp[htid * 4 + 1]) + ssp[htid * 4 + 2]) + ssp[htid * 4 + 3];
+          half_sync(half);
+        } else {
+          float rs[32];  // 1/rms of the chunk's tokens, read before any staging store
+          if (NORM) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {  // the 1/rms buffer has room past BN for the short chunk
+              const float4 v4 = *reinterpret_cast<const float4*>(rstd + c0 + j);
+              rs[j] = v4.x;
+              rs[j + 1] = v4.y;
+              rs[j + 2] = v4.z;
+              rs[j + 3] = v4.w;
+            }
+          }
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            float val = __uint_as_float(r[j]);
+            if (NORM) val *= rs[j];
+            if (EPI == kEpiStore) {
+              tH[j * kSH + row] = __float2half_rn(val);
+            } else {  // SwiGLU: lane l (l % 16 < 8) holds a gate row, lane l + 8 its up row
+              const float up = __shfl_down_sync(0xffffffffu, val, 8);
+              const __half hv = __float2half_rn(__fdividef(val, 1.f + __expf(-val)) * up);
+              if ((lane & 8) == 0) tH[j * kSG + (row >> 4) * 8 + (lane & 7)] = hv;
+            }
+          }
+          half_sync(half);
+          // coalesced 16-byte stores of the chunk's token rows
+          if (EPI == kEpiStore) {
+            for (int e = htid; e < nc * (kTileN / 8); e += 128) {
+              const int tk = e / (kTileN / 8);
+              const int u = e % (kTileN / 8);
+              const int m = m0 + c0 + tk;
+              if (m < p.M)
+                *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m) * p.ldy + n0 + u * 8) =
+                    *reinterpret_cast<const uint4*>(tH + tk * kSH + u * 8);
+            }
+          } else {
+            for (int e = htid; e < nc * 8; e += 128) {
+              const int tk = e >> 3;
+              const int u = e & 7;
+              const int m = m0 + c0 + tk;
+              if (m < p.M)
+                *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m) * p.ldy + n0 / 2 + u * 8) =
+                    *reinterpret_cast<const uint4*>(tH + tk * kSG + u * 8);
+            }
+          }
+          half_sync(half);  // staging free for the next chunk
+        }
+      }
+      // accumulator drained: hand it back to the MMA warp
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tmem_empty + acc);
     }
   }
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  tc_fence_before();
   __syncthreads();
   if (warp == 0)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
@@ -290,10 +404,18 @@ cudaError_t launch_gemm_tc(const CUtensorMap& map_a, const TcGemmArgs& args, int
   size_t smem = 0;
   const void* fn = tc_select(bn, epi, norm, &smem);
   if (!fn || args.N % kTileN != 0 || args.K % kTileK != 0) return cudaErrorInvalidValue;
+  static int sm_count = 0;
+  if (sm_count == 0) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sm_count, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess || sm_count <= 0) return e != cudaSuccess ? e : cudaErrorInvalidValue;
+  }
   CUtensorMap map = map_a;
   TcGemmArgs a = args;
   void* kargs[] = {&map, &a};
-  const dim3 grid(args.N / kTileN, (args.M + bn - 1) / bn);
+  const int tiles = (args.N / kTileN) * ((args.M + bn - 1) / bn);
+  const dim3 grid(static_cast<unsigned>(tiles < sm_count ? tiles : sm_count));
   return launch_ex(fn, grid, dim3(kTcThreads), smem, stream, pdl, kargs);
 }
 
