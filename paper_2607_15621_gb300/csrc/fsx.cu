@@ -83,6 +83,8 @@ struct fsx_handle_s {
   __half* hbuf = nullptr;
   float* part = nullptr;
   size_t part_bytes = 0;
+  float* gemm_part = nullptr;   // split-K partial tiles of the residual GEMMs
+  int* tile_count = nullptr;    // [sm_count] split arrivals per tile, zero between launches
   int* status = nullptr;
   TickArgs* d_args = nullptr;
   TickArgs h_args{};
@@ -288,6 +290,9 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     go.ldxo = d;
     go.ss_out = h->ss;
     go.ss_stride = h->ss_stride;
+    go.k_splits = fsx::gemm_tc_k_splits((d / 128) * ((M + bn - 1) / bn), HD / 64, h->sm_count);
+    go.part = h->gemm_part;
+    go.tile_count = h->tile_count;
     FSX_CUDA(mark(kClassWo, true));
     FSX_CUDA(fsx::launch_gemm_tc(h->map_o[bn_i], go, bn, fsx::kEpiResidual, false, st, pdl));
     FSX_CUDA(mark(kClassWo, false));
@@ -320,6 +325,9 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     gd.ldxo = d;
     gd.ss_out = h->ss;
     gd.ss_stride = h->ss_stride;
+    gd.k_splits = fsx::gemm_tc_k_splits((d / 128) * ((M + bn - 1) / bn), F / 64, h->sm_count);
+    gd.part = h->gemm_part;
+    gd.tile_count = h->tile_count;
     FSX_CUDA(mark(kClassDown, true));
     FSX_CUDA(fsx::launch_gemm_tc(h->map_h[bn_i], gd, bn, fsx::kEpiResidual, false, st, pdl));
     FSX_CUDA(mark(kClassDown, false));
@@ -416,7 +424,8 @@ void free_handle(fsx_handle_s* h) {
   for (cudaEvent_t e : h->tev) cudaEventDestroy(e);
   if (h->last_tick) cudaEventDestroy(h->last_tick);
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
-  void* bufs[] = {h->p_arena, h->p_x, h->p_counters, h->w_arena, h->params, h->x, h->x16, h->ss, h->qkv, h->o, h->hbuf, h->part, h->status, h->d_args,
+  void* bufs[] = {h->p_arena, h->p_x, h->p_counters, h->w_arena, h->params, h->x, h->x16, h->ss, h->qkv, h->o, h->hbuf, h->part,
+                  h->gemm_part, h->tile_count, h->status, h->d_args,
                   h->st_offsets, h->st_frames, h->st_waypoints};
   for (void* p : bufs)
     if (p) cudaFree(p);
@@ -660,6 +669,9 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
     part = std::max(part, fsx::attention_workspace_bytes(B, cfg->n_heads, attention_splits(h, B)));
   h->part_bytes = part;
   if (part) FSX_CUDA_H(cudaMalloc(&h->part, part));
+  FSX_CUDA_H(cudaMalloc(&h->gemm_part, fsx::gemm_tc_part_bytes(h->sm_count)));
+  FSX_CUDA_H(cudaMalloc(&h->tile_count, sizeof(int) * h->sm_count));
+  FSX_CUDA_H(cudaMemset(h->tile_count, 0, sizeof(int) * h->sm_count));
   FSX_CUDA_H(cudaMalloc(&h->status, sizeof(int)));
   FSX_CUDA_H(cudaMemset(h->status, 0, sizeof(int)));
   FSX_CUDA_H(cudaMalloc(&h->d_args, sizeof(TickArgs)));

@@ -107,6 +107,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
   const int KT = p.K / kTileK;
   const int tiles_n = p.N / kTileN;
   const int n_tiles = tiles_n * ((p.M + BN - 1) / BN);
+  const int KS = (EPI == kEpiResidual && p.k_splits > 1) ? p.k_splits : 1;
+  const int n_units = n_tiles * KS;  // unit u: tile u / KS, K steps [kt0(u), kt1(u))
+  auto kt0 = [&](int u) { return (u % KS) * KT / KS; };
+  auto kt1 = [&](int u) { return (u % KS + 1) * KT / KS; };
   constexpr int kAbytes = BN * kTileK * 2;
   constexpr uint32_t kTmemCols = tc_tmem_cols<BN>();
   // bounded wait that gives up at once after an earlier timeout of this CTA
@@ -140,36 +144,39 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(tmem_slot);
 
   if (warp == 0) {
-    // ---- producer (converged; lane 0 issues). Stage g of this CTA's stream is
-    // K step g % KT of its tile g / KT. Weights may stream before the previous
-    // kernel finished, the token tiles only after it.
-    const int my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - static_cast<int>(blockIdx.x)) / static_cast<int>(gridDim.x) + 1 : 0;
-    const int total = my_tiles * KT;
-    auto w_src = [&](int g) {
-      const int t = static_cast<int>(blockIdx.x) + (g / KT) * static_cast<int>(gridDim.x);
-      return p.w + (static_cast<size_t>(t % tiles_n) * KT + g % KT) * kWTileBytes;
+    // ---- producer (converged; lane 0 issues). Stage g of this CTA's stream runs
+    // over its units in order and over each unit's K steps. Weights may stream
+    // before the previous kernel finished, the token tiles only after it.
+    auto w_src = [&](int u, int kt) {
+      return p.w + (static_cast<size_t>((u / KS) % tiles_n) * KT + kt) * kWTileBytes;
     };
-    const int pre = total < kStages ? total : kStages;
-    if (lane == 0)
-      for (int g = 0; g < pre; ++g) {
-        mbar_arrive_expect_tx(full + g, kWTileBytes + kAbytes);
-        bulk_g2s(stages + g * tc_stage_bytes<BN>(), w_src(g), kWTileBytes, full + g);
-      }
+    if (lane == 0) {
+      int g = 0;
+      for (int u = blockIdx.x; u < n_units && g < kStages; u += gridDim.x)
+        for (int kt = kt0(u); kt < kt1(u) && g < kStages; ++kt, ++g) {
+          mbar_arrive_expect_tx(full + g, kWTileBytes + kAbytes);
+          bulk_g2s(stages + g * tc_stage_bytes<BN>(), w_src(u, kt), kWTileBytes, full + g);
+        }
+    }
     __syncwarp();
     pdl_wait();
-    for (int g = 0; g < total; ++g) {
-      const int s = g % kStages;
-      unsigned char* st = stages + s * tc_stage_bytes<BN>();
-      if (g >= kStages) wait(empty + s, static_cast<uint32_t>(((g / kStages) - 1) & 1));
-      if (lane == 0) {
-        const int t = static_cast<int>(blockIdx.x) + (g / KT) * static_cast<int>(gridDim.x);
-        if (g >= kStages) {
-          mbar_arrive_expect_tx(full + s, kWTileBytes + kAbytes);
-          bulk_g2s(st, w_src(g), kWTileBytes, full + s);
+    int total = 0;
+    for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+      const int m_tile = (u / KS) / tiles_n;
+      for (int kt = kt0(u); kt < kt1(u); ++kt, ++total) {
+        const int g = total;
+        const int s = g % kStages;
+        unsigned char* st = stages + s * tc_stage_bytes<BN>();
+        if (g >= kStages) wait(empty + s, static_cast<uint32_t>(((g / kStages) - 1) & 1));
+        if (lane == 0) {
+          if (g >= kStages) {
+            mbar_arrive_expect_tx(full + s, kWTileBytes + kAbytes);
+            bulk_g2s(st, w_src(u, kt), kWTileBytes, full + s);
+          }
+          tma_load_2d(st + kWTileBytes, &map_a, kt * kTileK, m_tile * BN, full + s);
         }
-        tma_load_2d(st + kWTileBytes, &map_a, (g % KT) * kTileK, (t / tiles_n) * BN, full + s);
+        __syncwarp();
       }
-      __syncwarp();
     }
     // after a timeout the MMA warp may have skipped its waits: let the copies still in
     // flight land (bounded) before the shared memory is released
@@ -192,12 +199,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
     constexpr uint32_t idesc = idesc_f16(kTileN, BN);
     int g = 0;
     int i = 0;
-    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+    for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++i) {
       const int acc = i & 1;
       if (i >= 2) wait(tmem_empty + acc, static_cast<uint32_t>(((i >> 1) - 1) & 1));
       tc_fence_after();
       const uint32_t d = tmem + static_cast<uint32_t>(acc * BN);
-      for (int kt = 0; kt < KT; ++kt, ++g) {
+      const int k_first = kt0(u);
+      for (int kt = k_first; kt < kt1(u); ++kt, ++g) {
         const int s = g % kStages;
         wait(full + s, static_cast<uint32_t>((g / kStages) & 1));
         tc_fence_after();
@@ -206,7 +214,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
           const uint32_t b_base = a_base + kWTileBytes;
 #pragma unroll
           for (int k = 0; k < kTileK / 16; ++k)
-            umma_f16(d, sw128_desc(a_base + k * 32), sw128_desc(b_base + k * 32), idesc, (kt > 0 || k > 0) ? 1u : 0u);
+            umma_f16(d, sw128_desc(a_base + k * 32), sw128_desc(b_base + k * 32), idesc,
+                     (kt > k_first || k > 0) ? 1u : 0u);
           umma_commit(empty + s);
         }
         __syncwarp();
@@ -228,11 +237,54 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
     constexpr int kSG = 64 + 8;      // fp16 row stride (SwiGLU: 64 columns per tile)
     __half* tH = reinterpret_cast<__half*>(stg + half * kStgHalfBytes);
     float* ssp = s_ssp + half * kEpiChunk * 4;
+    // x[m, n0 + row] += D[row, m] for the chunk's tokens: lanes hold consecutive columns,
+    // so every access of the warp is one contiguous 128-byte row piece; also the
+    // tokens' sums of x^2 over the tile's 128 columns
+    auto residual_chunk = [&](int tn_, int m0, int c0, int nc, uint32_t (&r)[32]) {
+      const int n0 = tn_ * kTileN;
+      const int n_ok = min(nc, p.M - (m0 + c0));  // valid tokens of the chunk
+      float* px = p.xo + static_cast<size_t>(m0 + c0) * p.ldxo + n0 + row;
+      __half* ph = p.xo16 + static_cast<size_t>(m0 + c0) * p.ldxo + n0 + row;
+      float x[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j)  // every load in flight before the first store
+        x[j] = j < n_ok ? __ldcg(px + static_cast<size_t>(j) * p.ldxo) : 0.f;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        x[j] += __uint_as_float(r[j]);
+        if (j < n_ok) {
+          px[static_cast<size_t>(j) * p.ldxo] = x[j];
+          ph[static_cast<size_t>(j) * p.ldxo] = __float2half_rn(x[j]);
+        }
+        x[j] = j < n_ok ? x[j] * x[j] : 0.f;
+      }
+      // 32 tokens x 32 lanes of x^2 -> lane l holds this quadrant's sum for token l
+#pragma unroll
+      for (int sh = 16; sh > 0; sh >>= 1) {
+        const bool upper = (lane & sh) != 0;
+#pragma unroll
+        for (int j = 0; j < sh; ++j) {
+          const float send = upper ? x[j] : x[j + sh];
+          const float keep = upper ? x[j + sh] : x[j];
+          x[j] = keep + __shfl_xor_sync(0xffffffffu, send, sh);
+        }
+      }
+      ssp[lane * 4 + q] = x[0];
+      half_sync(half);
+      if (htid < nc && p.ss_out != nullptr && m0 + c0 + htid < p.M)  // fixed quadrant order
+        p.ss_out[static_cast<size_t>(tn_) * p.ss_stride + m0 + c0 + htid] =
+            ((ssp[htid * 4 + 0] + ssp[htid * 4 + 1]) + ssp[htid * 4 + 2]) + ssp[htid * 4 + 3];
+      half_sync(half);
+    };
+    volatile int* s_last = reinterpret_cast<volatile int*>(tmem_slot + 2);
     int i = 0;
-    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+    for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++i) {
       const int acc = i & 1;
-      const int n0 = (t % tiles_n) * kTileN;
-      const int m0 = (t / tiles_n) * BN;
+      const int tile = u / KS;
+      const int split = u % KS;
+      const int t_n = tile % tiles_n;
+      const int n0 = t_n * kTileN;
+      const int m0 = (tile / tiles_n) * BN;
       float* rstd = s_rstd + acc * BN;
       if (NORM) {  // 1/rms of the tile's tokens from the per-128-column partial sums of x^2
         for (int tt = etid; tt < BN; tt += kEpiThreads) {
@@ -262,41 +314,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
           for (int j = 16; j < 32; ++j) r[j] = 0u;
         }
         if (EPI == kEpiResidual) {
-          // x[m, n0 + row] += D[row, m]: lanes hold consecutive columns, so every access
-          // of the warp is one contiguous 128-byte row piece
-          const int n_ok = min(nc, p.M - (m0 + c0));  // valid tokens of the chunk
-          float* px = p.xo + static_cast<size_t>(m0 + c0) * p.ldxo + n0 + row;
-          __half* ph = p.xo16 + static_cast<size_t>(m0 + c0) * p.ldxo + n0 + row;
-          float x[32];
+          if (KS == 1) {
+            residual_chunk(t_n, m0, c0, nc, r);
+          } else {  // this split's partial -> workspace ([tile][split][token][128 columns])
+            float* pp = p.part + (static_cast<size_t>(tile * KS + split) * BN + c0) * kTileN + row;
 #pragma unroll
-          for (int j = 0; j < 32; ++j)  // every load in flight before the first store
-            x[j] = j < n_ok ? __ldcg(px + static_cast<size_t>(j) * p.ldxo) : 0.f;
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            x[j] += __uint_as_float(r[j]);
-            if (j < n_ok) {
-              px[static_cast<size_t>(j) * p.ldxo] = x[j];
-              ph[static_cast<size_t>(j) * p.ldxo] = __float2half_rn(x[j]);
-            }
-            x[j] = j < n_ok ? x[j] * x[j] : 0.f;
+            for (int j = 0; j < 32; ++j)
+              if (j < nc) pp[static_cast<size_t>(j) * kTileN] = __uint_as_float(r[j]);
           }
-          // 32 tokens x 32 lanes of x^2 -> lane l holds this quadrant's sum for token l
-#pragma unroll
-          for (int sh = 16; sh > 0; sh >>= 1) {
-            const bool upper = (lane & sh) != 0;
-#pragma unroll
-            for (int j = 0; j < sh; ++j) {
-              const float send = upper ? x[j] : x[j + sh];
-              const float keep = upper ? x[j + sh] : x[j];
-              x[j] = keep + __shfl_xor_sync(0xffffffffu, send, sh);
-            }
-          }
-          ssp[lane * 4 + q] = x[0];
-          half_sync(half);
-          if (htid < nc && p.ss_out != nullptr && m0 + c0 + htid < p.M)  // fixed quadrant order
-            p.ss_out[static_cast<size_t>(t % tiles_n) * p.ss_stride + m0 + c0 + htid] =
-                ((ssp[htid * 4 + 0] + ssp[htid * 4 + 1]) + ssp[htid * 4 + 2]) + ssp[htid * 4 + 3];
-          half_sync(half);
         } else {
           float rs[32];  // 1/rms of the chunk's tokens, read before any staging store
           if (NORM) {
@@ -349,6 +374,62 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tmem_empty + acc);
+      if (EPI == kEpiResidual && KS > 1) {
+        // the last split of the tile to arrive adds all partials in split order
+        __threadfence();
+        epi_sync();
+        if (etid == 0) *s_last = atomicAdd(p.tile_count + tile, 1) == KS - 1;
+        epi_sync();
+        if (*s_last) {
+          __threadfence();
+          // warp ew takes tokens ew, ew + 12, ...; lane = 4-column group of the tile's 128
+          // columns; partials are summed in split order, 4 tokens' loads in flight at once
+          const int ew = etid >> 5;
+          constexpr int kEW = kEpiThreads / 32;
+          for (int tk0 = ew; tk0 < BN; tk0 += 4 * kEW) {
+            float4 acc4[4];
+#pragma unroll
+            for (int b = 0; b < 4; ++b) acc4[b] = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int sp = 0; sp < KS; ++sp) {
+              const float* pp = p.part + (static_cast<size_t>(tile * KS + sp) * BN) * kTileN + lane * 4;
+              float4 w4[4];
+#pragma unroll
+              for (int b = 0; b < 4; ++b) {
+                const int tk = tk0 + b * kEW;
+                w4[b] = tk < BN ? __ldcg(reinterpret_cast<const float4*>(pp + static_cast<size_t>(tk) * kTileN))
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+              }
+#pragma unroll
+              for (int b = 0; b < 4; ++b) {
+                acc4[b].x += w4[b].x;
+                acc4[b].y += w4[b].y;
+                acc4[b].z += w4[b].z;
+                acc4[b].w += w4[b].w;
+              }
+            }
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+              const int tk = tk0 + b * kEW;
+              const int m = m0 + tk;
+              float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+              const size_t idx = static_cast<size_t>(m) * p.ldxo + n0 + lane * 4;
+              if (tk < BN && m < p.M) {
+                const float4 x0 = __ldcg(reinterpret_cast<const float4*>(p.xo + idx));
+                x = make_float4(x0.x + acc4[b].x, x0.y + acc4[b].y, x0.z + acc4[b].z, x0.w + acc4[b].w);
+                *reinterpret_cast<float4*>(p.xo + idx) = x;
+                uint2 pk;
+                pk.x = pack_half2(x.x, x.y);
+                pk.y = pack_half2(x.z, x.w);
+                *reinterpret_cast<uint2*>(p.xo16 + idx) = pk;
+              }
+              const float ss = warp_sum(x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w);
+              if (lane == 0 && tk < BN && m < p.M && p.ss_out != nullptr)
+                p.ss_out[static_cast<size_t>(t_n) * p.ss_stride + m] = ss;
+            }
+          }
+          if (etid == 0) p.tile_count[tile] = 0;  // ready for the next launch
+        }
+      }
     }
   }
   tc_fence_before();
@@ -399,6 +480,17 @@ cudaError_t gemm_tc_set_attributes() {
   return cudaSuccess;
 }
 
+int gemm_tc_k_splits(int tiles, int KT, int sm_count) {
+  if (tiles <= 0 || tiles >= sm_count) return 1;
+  int ks = sm_count / tiles;                // all units in one wave
+  const int max_ks = KT / 4;                // at least 4 K steps (16 MMAs) per unit
+  if (ks > max_ks) ks = max_ks;
+  return ks < 1 ? 1 : ks;
+}
+
+// tiles x splits <= sm_count whenever splits > 1, and a partial tile is at most 128 x 256 fp32
+size_t gemm_tc_part_bytes(int sm_count) { return static_cast<size_t>(sm_count) * kTileN * 256 * sizeof(float); }
+
 cudaError_t launch_gemm_tc(const CUtensorMap& map_a, const TcGemmArgs& args, int bn, int epi, bool norm,
                            cudaStream_t stream, bool pdl) {
   size_t smem = 0;
@@ -414,8 +506,9 @@ cudaError_t launch_gemm_tc(const CUtensorMap& map_a, const TcGemmArgs& args, int
   CUtensorMap map = map_a;
   TcGemmArgs a = args;
   void* kargs[] = {&map, &a};
-  const int tiles = (args.N / kTileN) * ((args.M + bn - 1) / bn);
-  const dim3 grid(static_cast<unsigned>(tiles < sm_count ? tiles : sm_count));
+  if (a.k_splits > 1 && (epi != kEpiResidual || a.part == nullptr || a.tile_count == nullptr)) return cudaErrorInvalidValue;
+  const int units = (args.N / kTileN) * ((args.M + bn - 1) / bn) * (a.k_splits > 1 ? a.k_splits : 1);
+  const dim3 grid(static_cast<unsigned>(units < sm_count ? units : sm_count));
   return launch_ex(fn, grid, dim3(kTcThreads), smem, stream, pdl, kargs);
 }
 

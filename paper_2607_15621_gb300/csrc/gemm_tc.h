@@ -31,7 +31,20 @@ struct TcGemmArgs {
   int n_ss;
   int ss_stride;
   int* status;
+  // split K (kEpiResidual only): k_splits > 1 cuts each tile's K steps into k_splits
+  // near-equal ranges run by different CTAs; each writes its fp32 partial tile to
+  // `part` ([tile][split][BN tokens][128]) and the last of a tile's splits to arrive
+  // (counted in tile_count[tile], zero between launches) adds the partials in split
+  // order and applies the residual update.
+  int k_splits;
+  float* part;
+  int* tile_count;
 };
+
+// k splits for a residual GEMM with `tiles` output tiles of KT k steps on `sm_count` SMs
+int gemm_tc_k_splits(int tiles, int KT, int sm_count);
+// bytes of the split-K partial workspace that covers every GEMM of a handle
+size_t gemm_tc_part_bytes(int sm_count);
 
 cudaError_t gemm_tc_set_attributes();
 cudaError_t launch_gemm_tc(const CUtensorMap& map_a, const TcGemmArgs& args, int bn, int epi, bool norm,

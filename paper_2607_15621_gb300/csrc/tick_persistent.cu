@@ -9,7 +9,7 @@
 //     L2) -> the CTA's 96 rows of [W_q; W_k; W_v] for head h (32 q, 32 k, 32 v
 //     dims) on the tensor cores (tcgen05, accumulator in tensor memory) ->
 //     q, k_ae, v_ae pushed to all 4 CTAs -> Eq. 1 over a quarter of
-//     [K_vlm ; K_ae] per CTA -> the 4 split results merged in shared memory
+//     [K_vlm ; K_ae] per CTA -> the 4 fp32 split results merged in shared memory
 //     (log-sum-exp weights) -> the CTA's 128 output columns of o_h W_o^T
 //     (tcgen05) added into the next residual state with vector atomics
 //     (cluster 0 also adds the residual itself).
@@ -83,7 +83,7 @@ __host__ __device__ inline Smem smem_layout(int d) {
   s.ownv = o;      o += kTokTile * kQS * 2;    // own values
   o = (o + 1023) & ~1023;
   s.tile = o;      o += 2 * kKeyTile * kD * 2; // fp16 K|V tile; later the merged o_h, swizzled
-  s.recv = o;      o += kCl * kRowsPerRank * kD * 2;  // fp16 split partials of the rows this CTA merges
+  s.recv = o;      o += kCl * kRowsPerRank * kD * 4;  // fp32 split partials of the rows this CTA merges
   s.recv_lse = o;  o += kCl * kRowsPerRank * 4;
   s.total = o + 1024;                          // + alignment slack of the dynamic base
   return s;
@@ -117,6 +117,9 @@ __device__ __forceinline__ uint32_t cluster_addr(const void* local, int rank) {
 __device__ __forceinline__ void st_cluster_v4(uint32_t addr, uint4 v) {
   asm volatile("st.shared::cluster.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
                : "memory");
+}
+__device__ __forceinline__ void st_cluster_v2f(uint32_t addr, float a, float b) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1,%2};" ::"r"(addr), "f"(a), "f"(b) : "memory");
 }
 __device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
@@ -176,7 +179,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   __half* ownv = reinterpret_cast<__half*>(smem + L.ownv);
   unsigned char* hsl = smem + L.qbuf;  // phase B: swizzled [48 tokens x 64] SwiGLU slice of the cluster
   unsigned char* obuf = smem + L.tile;  // merged o_h, swizzled [48 tokens x 128]
-  __half* recv = reinterpret_cast<__half*>(smem + L.recv);
+  float* recv = reinterpret_cast<float*>(smem + L.recv);
   float* recv_lse = reinterpret_cast<float*>(smem + L.recv_lse);
   float* dstT = reinterpret_cast<float*>(smem + L.ownk);  // [48][kDS] fp32 output transpose (aliases ownk/ownv)
 
@@ -656,38 +659,29 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       attend(reinterpret_cast<const unsigned char*>(ownk + static_cast<size_t>(own_lo) * kQS),
              reinterpret_cast<const unsigned char*>(ownv + static_cast<size_t>(own_lo) * kQS), kQS * 2, own_n);
 
-    // --- merge the 4 splits: stage this split's normalised partial (fp16) and
-    // log-sum-exp locally, then send each row to the rank that owns it
-    __half* part = reinterpret_cast<__half*>(obuf);  // [48][kD] (tile area)
-    float* part_lse = reinterpret_cast<float*>(smem + L.lse);
+    // --- merge the 4 splits: every row's normalised fp32 partial and log-sum-exp go
+    // straight from the registers to the rank that owns the row
     if (warp < 6) {
       const int qr0 = qt * 16 + (lane >> 2);
       const int qr1 = qr0 + 8;
+      const int own0 = qr0 / kRowsPerRank;
+      const int own1 = qr1 / kRowsPerRank;
       const float inv0 = l_run[0] > 0.f ? 1.f / l_run[0] : 0.f;
       const float inv1 = l_run[1] > 0.f ? 1.f / l_run[1] : 0.f;
+      float* d0 = recv + (rank * kRowsPerRank + qr0 - own0 * kRowsPerRank) * kD;
+      float* d1 = recv + (rank * kRowsPerRank + qr1 - own1 * kRowsPerRank) * kD;
 #pragma unroll
       for (int n = 0; n < 8; ++n) {
         const int c = dh * 64 + n * 8 + 2 * (lane & 3);
-        *reinterpret_cast<uint32_t*>(part + qr0 * kD + c) = pack_half2(o_acc[n][0] * inv0, o_acc[n][1] * inv0);
-        *reinterpret_cast<uint32_t*>(part + qr1 * kD + c) = pack_half2(o_acc[n][2] * inv1, o_acc[n][3] * inv1);
+        st_cluster_v2f(cluster_addr(d0 + c, own0), o_acc[n][0] * inv0, o_acc[n][1] * inv0);
+        st_cluster_v2f(cluster_addr(d1 + c, own1), o_acc[n][2] * inv1, o_acc[n][3] * inv1);
       }
       if (dh == 0 && (lane & 3) == 0) {
-        part_lse[qr0] = l_run[0] > 0.f ? m_run[0] + log2f(l_run[0]) : -CUDART_INF_F;
-        part_lse[qr1] = l_run[1] > 0.f ? m_run[1] + log2f(l_run[1]) : -CUDART_INF_F;
+        st_cluster_f32(cluster_addr(recv_lse + rank * kRowsPerRank + qr0 - own0 * kRowsPerRank, own0),
+                       l_run[0] > 0.f ? m_run[0] + log2f(l_run[0]) : -CUDART_INF_F);
+        st_cluster_f32(cluster_addr(recv_lse + rank * kRowsPerRank + qr1 - own1 * kRowsPerRank, own1),
+                       l_run[1] > 0.f ? m_run[1] + log2f(l_run[1]) : -CUDART_INF_F);
       }
-    }
-    __syncthreads();
-    for (int i = tid; i < kTokTile * (kD / 8); i += kThr) {  // 48 rows x 16 units
-      const int row = i / (kD / 8);
-      const int u = i - row * (kD / 8);
-      const int owner = row / kRowsPerRank;
-      const __half* src = part + row * kD + u * 8;
-      st_cluster_v4(cluster_addr(recv + (rank * kRowsPerRank + row - owner * kRowsPerRank) * kD + u * 8, owner),
-                    *reinterpret_cast<const uint4*>(src));
-    }
-    if (tid < kTokTile) {
-      const int owner = tid / kRowsPerRank;
-      st_cluster_f32(cluster_addr(recv_lse + rank * kRowsPerRank + tid - owner * kRowsPerRank, owner), part_lse[tid]);
     }
     cluster.sync();
     // merged rows of o_h -> swizzled image in every partner's obuf (the W_o B operand)
@@ -705,13 +699,11 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
 #pragma unroll
           for (int s = 0; s < kCl; ++s) {
             const float w = exp2f(recv_lse[s * kRowsPerRank + rr] - mmax);
-            const uint2 pk = *reinterpret_cast<const uint2*>(recv + (s * kRowsPerRank + rr) * kD + c);
-            const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&pk.x));
-            const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&pk.y));
-            a0 += w * f0.x;
-            a1 += w * f0.y;
-            a2 += w * f1.x;
-            a3 += w * f1.y;
+            const float4 f = *reinterpret_cast<const float4*>(recv + (s * kRowsPerRank + rr) * kD + c);
+            a0 += w * f.x;
+            a1 += w * f.y;
+            a2 += w * f.z;
+            a3 += w * f.w;
             wsum += w;
           }
         }
