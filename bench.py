@@ -14,6 +14,7 @@ so no flush is needed between ticks.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -35,7 +36,9 @@ KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down", "persistent"]
 # kernel as it is now (profiles/ holds each summary with its command). A kernel that changed
 # after its capture gets no entry, so its traffic is reported as null.
 NCU_TRAFFIC = {
-    ("qkv", "bf16_b16_ragged"): 13.401088e6,                     # gemm_tc_bf16_b16_ragged.md
+    ("persistent", "bf16_b1_l224"): 792.98944e6 + 3.55968e6,     # persistent_tick_bf16_b1_l224.md
+    ("qkv", "bf16_b128_ragged"): 18.218752e6 + 71.825408e6,      # gemm_tc_bf16_b128_ragged.md
+    ("attention", "bf16_b128_ragged"): 2266.469e6 + 63.851776e6, # attn_splitkv_bf16_b128_ragged.md
 }
 
 
@@ -46,9 +49,13 @@ def parse():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--workload", default="bf16_b1_l224")
     ap.add_argument("--impl", default="fsx", choices=["fsx", "reference"])
-    ap.add_argument("--kernel-class", default="qkv", choices=KCLASS_NAMES)
+    ap.add_argument("--kernel-class", default=None, choices=KCLASS_NAMES,
+                    help="kernel timed for the roofline (default: the dominant one, i.e. the persistent tick "
+                         "for one vehicle and attention for a batch)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="expert layers (default: the workload's 32); fewer layers keep a profiling run's cache small")
     return ap.parse_args()
 
 
@@ -179,7 +186,7 @@ def main():
 
     from paper_2607_15621_gb300 import fsx, synth
     spec, lengths = workload_info(args.workload)
-    dims = synth.EXPERT
+    dims = synth.EXPERT if args.layers is None else dataclasses.replace(synth.EXPERT, n_layers=args.layers)
     dtype = spec["dtype"]
     B = len(lengths)
     w = synth.make_weights(dims, 0, dtype)
@@ -248,6 +255,8 @@ def main():
     kclass = args.kernel_class
     if ex.launches(B) == 1:  # single-launch persistent tick: the tick kernel is the dominant kernel
         kclass = "persistent"
+    elif kclass is None:  # batched ticks: Eq. 1 attention streams the cache and dominates
+        kclass = "attention"
     ex.set_kernel_timing(True, kclass)
     kt_ms, kt_n = [], 0
     for i in range(max(args.steps // 4, 5) + 2):
