@@ -108,7 +108,6 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
 
   const int split = blockIdx.x;
   const int h = blockIdx.y;
-  const int b = blockIdx.z;
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const int lane = tid & 31;
@@ -116,6 +115,7 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
 
   pdl_launch_dependents();
   pdl_wait();
+  const int b = p.order != nullptr ? p.order[blockIdx.z] : static_cast<int>(blockIdx.z);
   // The CTAs of a merge cluster read each other's shared memory, so they must
   // all stay; a raised status is honoured per vehicle below instead.
   if (!CM && *reinterpret_cast<volatile int*>(p.status) != 0) return;

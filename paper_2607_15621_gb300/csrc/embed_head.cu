@@ -3,7 +3,9 @@
 // embed: x_b = [E_act ; F_b] + P_pos into the fp32 residual stream; block 0
 //        also checks the cache offsets (non-decreasing, within capacity) and
 //        raises the device status word, which turns the rest of the tick
-//        into no-ops.
+//        into no-ops. Block b < B also ranks vehicle b by cache length, so the
+//        attention launches can start the longest caches first (a schedule
+//        only: every (vehicle, head) computes the same result in any order).
 // head:  waypoint j of vehicle b = W_h RMSNorm(x_{b,j}; g_f) + b_h, fp32.
 #include "device_util.cuh"
 #include "kernels.h"
@@ -26,9 +28,27 @@ __global__ void embed_kernel(const EmbedArgs a) {
     ok = ok && off[a.B] <= a.max_total;
     if (!ok) set_status(a.status, kStatusDeviceArg);
   }
+  __shared__ float s_part[4];
+  __shared__ int s_cnt[4];
+  if (a.order != nullptr && row < a.B) {  // rank of vehicle `row`: longer caches first, ties by index
+    const int64_t* off = a.targs->offsets;
+    const int64_t len = off[row + 1] - off[row];
+    int cnt = 0;
+    for (int j = threadIdx.x; j < a.B; j += blockDim.x) {
+      const int64_t lj = off[j + 1] - off[j];
+      cnt += (lj > len || (lj == len && j < row)) ? 1 : 0;
+    }
+    for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+    if ((threadIdx.x & 31) == 0) s_cnt[threadIdx.x >> 5] = cnt;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int r = 0;
+      for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) r += s_cnt[w];
+      a.order[r] = row;
+    }
+  }
   float* xr = a.x + static_cast<size_t>(row) * a.d;
   const float* pos = a.pos_emb + static_cast<size_t>(t) * a.d;
-  __shared__ float s_part[4];
   for (int c = threadIdx.x; c < a.d; c += blockDim.x) {
     float v;
     if (t < a.n_action) {

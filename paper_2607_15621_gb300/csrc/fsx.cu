@@ -85,6 +85,7 @@ struct fsx_handle_s {
   size_t part_bytes = 0;
   float* gemm_part = nullptr;   // split-K partial tiles of the residual GEMMs
   int* tile_count = nullptr;    // [sm_count] split arrivals per tile, zero between launches
+  int* order = nullptr;         // [max_batch] vehicles by decreasing cache length (attention schedule)
   int* status = nullptr;
   TickArgs* d_args = nullptr;
   TickArgs h_args{};
@@ -224,6 +225,7 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
   ea.x16 = h->x16;
   ea.ss = h->ss;
   ea.ss_stride = h->ss_stride;
+  ea.order = h->order;
   ea.status = h->status;
   FSX_CUDA(fsx::launch_embed(ea, st, pdl));
 
@@ -269,6 +271,7 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     a.lse = nullptr;
     a.part_o = h->part;
     a.part_lse = h->part + static_cast<size_t>(B) * c.n_heads * S * fsx::kTokTile * fsx::kHeadDim;
+    a.order = h->order;
     a.status = h->status;
     FSX_CUDA(mark(kClassAttn, true));
     FSX_CUDA(fsx::launch_attention(a, B, c.cache_dtype, st, pdl));
@@ -425,7 +428,7 @@ void free_handle(fsx_handle_s* h) {
   if (h->last_tick) cudaEventDestroy(h->last_tick);
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
   void* bufs[] = {h->p_arena, h->p_x, h->p_counters, h->w_arena, h->params, h->x, h->x16, h->ss, h->qkv, h->o, h->hbuf, h->part,
-                  h->gemm_part, h->tile_count, h->status, h->d_args,
+                  h->gemm_part, h->tile_count, h->order, h->status, h->d_args,
                   h->st_offsets, h->st_frames, h->st_waypoints};
   for (void* p : bufs)
     if (p) cudaFree(p);
@@ -672,6 +675,7 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
   FSX_CUDA_H(cudaMalloc(&h->gemm_part, fsx::gemm_tc_part_bytes(h->sm_count)));
   FSX_CUDA_H(cudaMalloc(&h->tile_count, sizeof(int) * h->sm_count));
   FSX_CUDA_H(cudaMemset(h->tile_count, 0, sizeof(int) * h->sm_count));
+  FSX_CUDA_H(cudaMalloc(&h->order, sizeof(int) * cfg->max_batch));
   FSX_CUDA_H(cudaMalloc(&h->status, sizeof(int)));
   FSX_CUDA_H(cudaMemset(h->status, 0, sizeof(int)));
   FSX_CUDA_H(cudaMalloc(&h->d_args, sizeof(TickArgs)));

@@ -49,6 +49,7 @@ struct AttnArgs {
   float* lse;                 // optional [B, H, n_q] natural log
   float* part_o;              // [B, H, S, 48, 128] when n_splits > 1
   float* part_lse;            // [B, H, S, 48]   (log2 domain)
+  const int* order;           // optional [B]: CTA row z works on vehicle order[z] (longest cache first)
   int* status;
 };
 
@@ -70,6 +71,7 @@ struct EmbedArgs {
   __half* x16;            // fp16 copy of x
   float* ss;              // per-row sums of x^2 over 128-column groups, [d/128][ss_stride]
   int ss_stride;
+  int* order;             // optional [B]: vehicles by decreasing cache length (ties by index)
   int* status;
 };
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t stream, bool pdl);
