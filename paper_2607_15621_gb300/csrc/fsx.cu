@@ -594,15 +594,17 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
         for (int cta = 0; cta < n_b * fsx::kPersistCluster; ++cta) {
           const int cl = cta / fsx::kPersistCluster, rank = cta % fsx::kPersistCluster;
           unsigned char* b = base + h->p_b_offset + static_cast<size_t>(cta) * h->p_b_cta;
-          // rows 0-15: gate columns 64 cl + 16 rank + r; rows 16-31: the matching up columns
+          // the cluster's 128 gate/up rows over this rank's K quarter (columns 128 rank ..):
+          // rows 32s + i, i < 16: gate column 64 cl + 16 s + i; i >= 16: the matching up column
           pack_sw128([&](int r) -> const float* {
-            const int col = cl * 64 + rank * 16 + r % 16;
-            return (r < 16 ? wg : wu) + static_cast<size_t>(col) * d;
-          }, 32, d, g2, b);
+            const int s_ = r / 32, i = r % 32;
+            const int col = cl * 64 + s_ * 16 + i % 16;
+            return (i < 16 ? wg : wu) + static_cast<size_t>(col) * d + rank * 128;
+          }, 128, 128, g2 + rank * 128, b);
           // 128 output columns x this cluster's 64 SwiGLU inputs
           pack_sw128([&](int r) -> const float* {
             return wd + static_cast<size_t>(rank * 128 + r) * F + cl * 64;
-          }, 128, 64, nullptr, b + 32 * 128 * (d / 64));
+          }, 128, 64, nullptr, b + 128 * 128 * 2);  // after the two gate/up K slices
         }
       };
       const int n_threads = std::max(1, std::min<int>(16, static_cast<int>(std::thread::hardware_concurrency())));

@@ -14,9 +14,12 @@
 //     (tcgen05) added into the next residual state with vector atomics
 //     (cluster 0 also adds the residual itself).
 //   phase B (clusters 0 .. F/64-1; cluster c owns SwiGLU columns 64c..64c+63):
-//     x -> RMSNorm -> the CTA's 16 SwiGLU columns (16 gate rows, then the
-//     matching 16 up rows; tcgen05) -> h pushed to all 4 CTAs -> the CTA's 128
-//     output columns of h W_d^T (tcgen05) added into the next residual state.
+//     each CTA reads only its 128 columns of x; the per-token sums of x^2 are
+//     completed across the cluster -> RMSNorm of those columns -> the cluster's
+//     128 gate/up rows over this CTA's K quarter (tcgen05) -> the partials
+//     reduce-scattered so that each CTA sums its 16 gate + 16 up rows -> h
+//     pushed to all 4 CTAs -> the CTA's 128 output columns of h W_d^T
+//     (tcgen05) added into the next residual state.
 // The residual stream rotates through three fp32 buffers: a phase reads one,
 // accumulates into the next (zeroed one phase earlier) and zeroes the third.
 //
@@ -28,9 +31,8 @@
 // layers. A layer takes 12 ring positions (6 of QKV, 2 of W_o, 2 of gate/up,
 // 1 of W_d and one empty position; CTAs without SwiGLU work leave positions
 // 8-11 empty), so the QKV images of every layer start at slot 0. The MMAs run
-// with M = 128: the 96-row QKV and 32-row gate/up images are padded with
-// whatever follows them in shared memory, and the rows that produces are never
-// read. The layer's backbone cache rows are prefetched into L2 at the start of
+// with M = 128: the 96-row QKV images are padded with whatever follows them in
+// shared memory, and the accumulator rows that produces are never read. The layer's backbone cache rows are prefetched into L2 at the start of
 // the layer and converted bf16/fp32 -> fp16 while staging 32-key tiles.
 #include <cooperative_groups.h>
 #include <math_constants.h>
@@ -57,7 +59,6 @@ constexpr int kQS = kD + 8;            // fp16 row stride of q / own k / own v (
 constexpr int kDS = 128 + 4;           // fp32 row stride of the output transpose buffer
 constexpr int kRowsPerRank = kTokTile / kCl;  // 12
 constexpr int kQkvAtom = 3 * 32 * 128;        // one 64-wide K slice of the CTA's 96 QKV rows (12 KB)
-constexpr int kGuAtom = 32 * 128;             // one K slice of the 32 gate/up rows (4 KB)
 constexpr int kActAtom = kTokTile * 128;      // one K slice of the 48 token rows (6 KB)
 constexpr uint32_t kTmemCols = 64;            // accumulator: 128 lanes x 48 fp32 columns
 constexpr uint32_t kIdesc = idesc_f16(128, kTokTile);
@@ -759,49 +760,87 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         const int e1 = static_cast<int>(static_cast<long long>(n_elem) * (cta + 1) / n_b_ctas);
         for (int e = e0 + tid; e < e1; e += kThr) __stcg(Xc + e, 0.f);
       }
-      load_normalized(Xm);
-      // gate/up: D[32 (+96 unused) rows x 48 tokens], 4 KB K slices in slots 2, 3
+      // --- RMSNorm split along K: this rank reads only its 128 columns of x, sends its
+      // per-token partial sums of x^2 to every CTA of the cluster, and normalises its
+      // columns into the first two K slices of the activation image
+      float* gss = dstT;  // [4 ranks][48] partial sums of x^2 (dstT is idle until W_d)
+      constexpr int kRowsPerWarp = kTokTile / (kThr / 32);  // 6
+      float4 xv[kRowsPerWarp];
+#pragma unroll
+      for (int i = 0; i < kRowsPerWarp; ++i) {
+        const int r = warp + 8 * i;
+        xv[i] = r < T ? ld_cg4(Xm + static_cast<size_t>(r) * d + rank * 128 + lane * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int i = 0; i < kRowsPerWarp; ++i) {
+        const int r = warp + 8 * i;
+        const float ps = warp_sum(xv[i].x * xv[i].x + xv[i].y * xv[i].y + xv[i].z * xv[i].z + xv[i].w * xv[i].w);
+        if (r < T && lane < kCl) st_cluster_f32(cluster_addr(gss + rank * kTokTile + r, lane), ps);
+      }
+      cluster.sync();  // every rank's partial sums arrived
+#pragma unroll
+      for (int i = 0; i < kRowsPerWarp; ++i) {
+        const int r = warp + 8 * i;
+        if (r < T) {
+          const float ss = ((gss[r] + gss[kTokTile + r]) + gss[2 * kTokTile + r]) + gss[3 * kTokTile + r];
+          const float rstd = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
+          uint2 pk;
+          pk.x = pack_half2(xv[i].x * rstd, xv[i].y * rstd);
+          pk.y = pack_half2(xv[i].z * rstd, xv[i].w * rstd);
+          *reinterpret_cast<uint2*>(act + sw128_offset(kTokTile, r, lane * 4)) = pk;
+        }
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // visible to the tensor core
+      __syncthreads();
+      // gate/up over this rank's K quarter: D[128 rows x 48 tokens], rows 32s..32s+31 =
+      // the 16 gate and 16 up rows of rank s's SwiGLU columns (K slices in slots 2, 3)
       if (warp == 0) {
         tc_fence_after();
-        for (int a = 0; a < d / 64; ++a) {
-          const int pos = kPersistAChunks + (a * kGuAtom) / kSlotBytes;
-          bool ok = true;
-          if ((a * kGuAtom) % kSlotBytes == 0) ok = wait_chunk(q0 + pos);
-          ok = ok && *abort == 0;
-          if (ok && lane == 0) mma_slice(ring_a + 2 * kSlotBytes + a * kGuAtom, act_a + a * kActAtom, a == 0);
+        for (int a = 0; a < 2; ++a) {
+          const bool ok = wait_chunk(q0 + kPersistAChunks + a);
+          if (ok && lane == 0) mma_slice(ring_a + (2 + a) * kSlotBytes, act_a + a * kActAtom, a == 0);
           __syncwarp();
         }
         if (lane == 0) umma_commit(mma_bar);
         __syncwarp();
       }
       wait_mma();
-      // accumulator rows 0-15: gate of columns 16 rank + r, rows 16-31: the matching
-      // up rows. Warps 0 and 4 (the ones that reach TMEM lanes 0-31) copy them out
-      // as [32 rows][49] fp32; then every thread forms h = silu(gate) * up.
-      float* graw = dstT;
-      constexpr int kGS = kTokTile + 1;
-      if ((warp & 3) == 0) {
-        for (int c0 = warp == 0 ? 0 : 32; c0 < (warp == 0 ? 32 : 48); c0 += 16) {
+      // reduce-scatter of the K partials: rows 32s..32s+31 go to rank s as
+      // recv[this rank][row][48 tokens] (fp32)
+      {
+        const int q = warp & 3;
+        const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16);
+        float* dst = recv + (rank * 32 + lane) * kTokTile;
+        for (int c0 = warp < 4 ? 0 : 32; c0 < (warp < 4 ? 32 : 48); c0 += 16) {
           float v[16];
           __syncwarp();
-          tmem_ld16(tmem + static_cast<uint32_t>(c0), v);
+          tmem_ld16(taddr + static_cast<uint32_t>(c0), v);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) graw[lane * kGS + c0 + j] = v[j];
+          for (int j = 0; j < 16; j += 4)
+            st_cluster_v4(cluster_addr(dst + c0 + j, q),
+                          make_uint4(__float_as_uint(v[j]), __float_as_uint(v[j + 1]), __float_as_uint(v[j + 2]),
+                                     __float_as_uint(v[j + 3])));
         }
-      }
-      __syncthreads();
-      for (int i = tid; i < kTokTile * 16; i += kThr) {
-        const int t = i >> 4;
-        const int cc = i & 15;
-        const float g = graw[cc * kGS + t];
-        const float u = graw[(16 + cc) * kGS + t];
-        *reinterpret_cast<__half*>(hsl + sw128_offset(kTokTile, t, rank * 16 + cc)) =
-            __float2half_rn(__fdividef(g, 1.f + __expf(-g)) * u);
       }
       tc_fence_before();
       __syncthreads();
       if (tid == 0)  // slots 2, 3 free: next layer's QKV
         for (int i = 2; i < 4; ++i) issue(q0 + kLayerChunks + i);
+      cluster.sync();  // every rank's partials of this rank's rows arrived
+      // h = silu(gate) * up for this rank's 16 SwiGLU columns, partials summed in rank order
+      for (int i = tid; i < kTokTile * 16; i += kThr) {
+        const int t = i >> 4;
+        const int cc = i & 15;
+        float g = 0.f, u = 0.f;
+#pragma unroll
+        for (int src = 0; src < kCl; ++src) {
+          g += recv[(src * 32 + cc) * kTokTile + t];
+          u += recv[(src * 32 + 16 + cc) * kTokTile + t];
+        }
+        *reinterpret_cast<__half*>(hsl + sw128_offset(kTokTile, t, rank * 16 + cc)) =
+            __float2half_rn(__fdividef(g, 1.f + __expf(-g)) * u);
+      }
+      __syncthreads();
       // this rank's 16 columns (two 16-byte units per token row) to the partners
       for (int i = tid; i < kTokTile * 2 * (kCl - 1); i += kThr) {
         const int peer_i = i / (kTokTile * 2);
