@@ -276,7 +276,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
             ((ssp[htid * 4 + 0] + ssp[htid * 4 + 1]) + ssp[htid * 4 + 2]) + ssp[htid * 4 + 3];
       half_sync(half);
     };
-    volatile int* s_last = reinterpret_cast<volatile int*>(tmem_slot + 2);
     int i = 0;
     for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++i) {
       const int acc = i & 1;
@@ -375,60 +374,77 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
       __syncwarp();
       if (lane == 0) mbar_arrive(tmem_empty + acc);
       if (EPI == kEpiResidual && KS > 1) {
-        // the last split of the tile to arrive adds all partials in split order
+        // every split of the tile waits until all KS partials are written (the grid holds
+        // at most one CTA per SM and never more CTAs than SMs, so all splits are resident),
+        // then adds the partials of its own slice of tokens in split order
         __threadfence();
         epi_sync();
-        if (etid == 0) *s_last = atomicAdd(p.tile_count + tile, 1) == KS - 1;
-        epi_sync();
-        if (*s_last) {
-          __threadfence();
-          // warp ew takes tokens ew, ew + 12, ...; lane = 4-column group of the tile's 128
-          // columns; partials are summed in split order, 4 tokens' loads in flight at once
-          const int ew = etid >> 5;
-          constexpr int kEW = kEpiThreads / 32;
-          for (int tk0 = ew; tk0 < BN; tk0 += 4 * kEW) {
-            float4 acc4[4];
-#pragma unroll
-            for (int b = 0; b < 4; ++b) acc4[b] = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int sp = 0; sp < KS; ++sp) {
-              const float* pp = p.part + (static_cast<size_t>(tile * KS + sp) * BN) * kTileN + lane * 4;
-              float4 w4[4];
-#pragma unroll
-              for (int b = 0; b < 4; ++b) {
-                const int tk = tk0 + b * kEW;
-                w4[b] = tk < BN ? __ldcg(reinterpret_cast<const float4*>(pp + static_cast<size_t>(tk) * kTileN))
-                                : make_float4(0.f, 0.f, 0.f, 0.f);
-              }
-#pragma unroll
-              for (int b = 0; b < 4; ++b) {
-                acc4[b].x += w4[b].x;
-                acc4[b].y += w4[b].y;
-                acc4[b].z += w4[b].z;
-                acc4[b].w += w4[b].w;
-              }
-            }
-#pragma unroll
-            for (int b = 0; b < 4; ++b) {
-              const int tk = tk0 + b * kEW;
-              const int m = m0 + tk;
-              float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
-              const size_t idx = static_cast<size_t>(m) * p.ldxo + n0 + lane * 4;
-              if (tk < BN && m < p.M) {
-                const float4 x0 = __ldcg(reinterpret_cast<const float4*>(p.xo + idx));
-                x = make_float4(x0.x + acc4[b].x, x0.y + acc4[b].y, x0.z + acc4[b].z, x0.w + acc4[b].w);
-                *reinterpret_cast<float4*>(p.xo + idx) = x;
-                uint2 pk;
-                pk.x = pack_half2(x.x, x.y);
-                pk.y = pack_half2(x.z, x.w);
-                *reinterpret_cast<uint2*>(p.xo16 + idx) = pk;
-              }
-              const float ss = warp_sum(x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w);
-              if (lane == 0 && tk < BN && m < p.M && p.ss_out != nullptr)
-                p.ss_out[static_cast<size_t>(t_n) * p.ss_stride + m] = ss;
+        if (etid == 0 && *abort == 0) {
+          atomicAdd(p.tile_count + tile, 1);
+          const unsigned long long t0 = global_timer_ns();
+          for (uint32_t it = 0;; ++it) {
+            int v;
+            asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p.tile_count + tile) : "memory");
+            if (v >= KS) break;
+            if ((it & 63u) == 63u && global_timer_ns() - t0 > kWaitLimitNs) {
+              set_status(p.status, kStatusTimeout);
+              *abort = 1;
+              break;
             }
           }
-          if (etid == 0) p.tile_count[tile] = 0;  // ready for the next launch
         }
+        epi_sync();
+        __threadfence();
+        const int tk_lo = split * BN / KS;
+        const int tk_hi = (split + 1) * BN / KS;
+        // warp ew takes tokens tk_lo + ew, + 12, ...; lane = 4-column group of the tile's
+        // 128 columns; 4 tokens' loads in flight at once
+        const int ew = etid >> 5;
+        constexpr int kEW = kEpiThreads / 32;
+        for (int tk0 = tk_lo + ew; tk0 < tk_hi; tk0 += 4 * kEW) {
+          float4 acc4[4];
+#pragma unroll
+          for (int bb = 0; bb < 4; ++bb) acc4[bb] = make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int sp = 0; sp < KS; ++sp) {
+            const float* pp = p.part + (static_cast<size_t>(tile * KS + sp) * BN) * kTileN + lane * 4;
+            float4 w4[4];
+#pragma unroll
+            for (int bb = 0; bb < 4; ++bb) {
+              const int tk = tk0 + bb * kEW;
+              w4[bb] = tk < tk_hi ? __ldcg(reinterpret_cast<const float4*>(pp + static_cast<size_t>(tk) * kTileN))
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int bb = 0; bb < 4; ++bb) {
+              acc4[bb].x += w4[bb].x;
+              acc4[bb].y += w4[bb].y;
+              acc4[bb].z += w4[bb].z;
+              acc4[bb].w += w4[bb].w;
+            }
+          }
+#pragma unroll
+          for (int bb = 0; bb < 4; ++bb) {
+            const int tk = tk0 + bb * kEW;
+            const int m = m0 + tk;
+            float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+            const size_t idx = static_cast<size_t>(m) * p.ldxo + n0 + lane * 4;
+            if (tk < tk_hi && m < p.M) {
+              const float4 x0 = __ldcg(reinterpret_cast<const float4*>(p.xo + idx));
+              x = make_float4(x0.x + acc4[bb].x, x0.y + acc4[bb].y, x0.z + acc4[bb].z, x0.w + acc4[bb].w);
+              *reinterpret_cast<float4*>(p.xo + idx) = x;
+              uint2 pk;
+              pk.x = pack_half2(x.x, x.y);
+              pk.y = pack_half2(x.z, x.w);
+              *reinterpret_cast<uint2*>(p.xo16 + idx) = pk;
+            }
+            const float ss = warp_sum(x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w);
+            if (lane == 0 && tk < tk_hi && m < p.M && p.ss_out != nullptr)
+              p.ss_out[static_cast<size_t>(t_n) * p.ss_stride + m] = ss;
+          }
+        }
+        // departures: the last split to leave resets the counter for the next launch
+        epi_sync();
+        if (etid == 0 && atomicAdd(p.tile_count + tile, 1) == 2 * KS - 1) p.tile_count[tile] = 0;
       }
     }
   }

@@ -32,10 +32,11 @@ struct TcGemmArgs {
   int ss_stride;
   int* status;
   // split K (kEpiResidual only): k_splits > 1 cuts each tile's K steps into k_splits
-  // near-equal ranges run by different CTAs; each writes its fp32 partial tile to
-  // `part` ([tile][split][BN tokens][128]) and the last of a tile's splits to arrive
-  // (counted in tile_count[tile], zero between launches) adds the partials in split
-  // order and applies the residual update.
+  // near-equal ranges run by different CTAs (never more units than SMs, one CTA per
+  // SM, so all are resident); each writes its fp32 partial tile to `part`
+  // ([tile][split][BN tokens][128]), waits until the tile's k_splits partials are
+  // there (tile_count[tile], zero between launches), and adds them in split order
+  // for its 1/k_splits share of the tile's tokens.
   int k_splits;
   float* part;
   int* tile_count;
