@@ -333,13 +333,29 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
               rs[j + 3] = v4.w;
             }
           }
+          if (EPI == kEpiStore) {
+            // token pairs (j, j + 1): the even lane packs columns (row, row + 1) of token j,
+            // the odd lane columns (row - 1, row) of token j + 1 -- one two-value fp16
+            // conversion and one 4-byte store per pair instead of two of each
+            const bool odd = (lane & 1) != 0;
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
+            for (int j = 0; j < 32; j += 2) {
+              float a = __uint_as_float(r[j]);
+              float b = __uint_as_float(r[j + 1]);
+              if (NORM) {
+                a *= rs[j];
+                b *= rs[j + 1];
+              }
+              const float other = __shfl_xor_sync(0xffffffffu, odd ? a : b, 1);
+              const __half2 h2 = odd ? __floats2half2_rn(other, b) : __floats2half2_rn(a, other);
+              *reinterpret_cast<__half2*>(tH + (odd ? (j + 1) * kSH + row - 1 : j * kSH + row)) = h2;
+            }
+          }
+#pragma unroll
+          for (int j = 0; j < 32 && EPI == kEpiSwiglu; ++j) {
             float val = __uint_as_float(r[j]);
             if (NORM) val *= rs[j];
-            if (EPI == kEpiStore) {
-              tH[j * kSH + row] = __float2half_rn(val);
-            } else {  // SwiGLU: lane l (l % 16 < 8) holds a gate row, lane l + 8 its up row
+            {  // SwiGLU: lane l (l % 16 < 8) holds a gate row, lane l + 8 its up row
               const float up = __shfl_down_sync(0xffffffffu, val, 8);
               const __half hv = __float2half_rn(__fdividef(val, 1.f + __expf(-val)) * up);
               if ((lane & 8) == 0) tH[j * kSG + (row >> 4) * 8 + (lane & 7)] = hv;
