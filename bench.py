@@ -66,6 +66,18 @@ def dist_env():
     return world, rank, local
 
 
+def max_over_ranks(value: float, device=None) -> float:
+    """Largest `value` over the ranks of the default process group (the value itself
+    when no group is initialised): the job's time is its slowest rank's time."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -165,7 +177,9 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / cb["value"],
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded)",
-            "config": {"workload": args.workload, "B": 1, "cache_len": int(lengths[0]), "layers": 32},
+            "config": {"workload": args.workload, "B": int(len(lengths)), "cache_len": [int(x) for x in lengths[:4]],
+                       "layers": 32, "parallelism": f"replicas x{world}",
+                       "sample": "vehicle 0 per step; vehicles are independent, so vehicle-ticks/s is per vehicle"},
             "cpu_baseline": cb,
             "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
@@ -227,11 +241,7 @@ def main():
     clocks = stop_clock_sampler(proc, fh, clock_path)
     if ex.status(stream) != fsx.FSX_OK:
         raise RuntimeError("device status set during the timed region")
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, dev)
     ms_per_step = ms / args.steps
     value = world * B * args.steps / (ms / 1e3)
 
@@ -248,6 +258,7 @@ def main():
         ex.tick_host(k, v, off_h.numpy(), frames_h, out_h.numpy(), stream)
     e2e_s = time.perf_counter() - t0
     barrier()
+    e2e_s = max_over_ranks(e2e_s, dev)
     h2d = frames_h.numel() * frames_h.element_size() + off_h.numel() * 8
     d2h = out_h.numel() * 4
 
