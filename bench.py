@@ -36,9 +36,9 @@ KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down", "persistent"]
 # kernel as it is now (profiles/ holds each summary with its command). A kernel that changed
 # after its capture gets no entry, so its traffic is reported as null.
 NCU_TRAFFIC = {
-    ("persistent", "bf16_b1_l224"): 792.98944e6 + 3.55968e6,     # persistent_tick_bf16_b1_l224.md
-    ("qkv", "bf16_b128_ragged"): 18.218752e6 + 71.825408e6,      # gemm_tc_bf16_b128_ragged.md
-    ("attention", "bf16_b128_ragged"): 2266.469e6 + 63.851776e6, # attn_splitkv_bf16_b128_ragged.md
+    ("persistent", "bf16_b1_l224"): 793.150976e6 + 3.595776e6,   # persistent_tick_bf16_b1_l224.md
+    ("qkv", "bf16_b128_ragged"): 18.229504e6 + 71.913728e6,      # gemm_tc_bf16_b128_ragged.md
+    ("attention", "bf16_b128_ragged"): 2262.161e6 + 45.69216e6,  # attn_splitkv_bf16_b128_ragged.md
 }
 
 
