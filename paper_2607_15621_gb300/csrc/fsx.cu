@@ -233,6 +233,10 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
   // token tile of the tensor-core GEMMs: 48 for one vehicle, then 128 / 256
   const int bn_i = M <= 48 ? 0 : (M <= 1024 ? 1 : 2);
   const int bn = bn_i == 0 ? 48 : (bn_i == 1 ? 128 : 256);
+  // QKV (N = 12288) has tiles to spare: 256-token tiles halve its MMA instructions (one
+  // tcgen05.mma costs the same for any N up to 256) whenever M exceeds one 48-token tile
+  const int bq_i = M <= 48 ? 0 : 2;
+  const int bq = bq_i == 0 ? 48 : 256;
   const int S = attention_splits(h, B);
 
   for (int l = 0; l < c.n_layers; ++l) {
@@ -249,7 +253,7 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     g.n_ss = d / 128;
     g.ss_stride = h->ss_stride;
     FSX_CUDA(mark(kClassQkv, true));
-    FSX_CUDA(fsx::launch_gemm_tc(h->map_x16[bn_i], g, bn, fsx::kEpiStore, true, st, pdl));
+    FSX_CUDA(fsx::launch_gemm_tc(h->map_x16[bq_i], g, bq, fsx::kEpiStore, true, st, pdl));
     FSX_CUDA(mark(kClassQkv, false));
 
     // Eq. 1 over [cache_l ; own]
