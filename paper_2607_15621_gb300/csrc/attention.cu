@@ -444,35 +444,42 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
 }
 
 // Merge of the split partials of one (vehicle, head): 128 threads = 128 dims.
-__global__ void __launch_bounds__(kD) attn_combine_kernel(const AttnArgs p) {
+// Merge of the split partials: one warp per (head, vehicle, query), lane = 4 dims; the
+// splits are added in split order.
+__global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs p) {
   const int h = blockIdx.x;
   const int b = blockIdx.y;
-  const int d = threadIdx.x;
+  const int qi = blockIdx.z * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
   const int H = p.n_heads;
   const int S = p.n_splits;
   pdl_launch_dependents();
   pdl_wait();
-  if (*reinterpret_cast<volatile int*>(p.status) != 0) return;
+  if (*reinterpret_cast<volatile int*>(p.status) != 0 || qi >= p.n_q) return;
   const size_t base = (static_cast<size_t>(b) * H + h) * S;
-  for (int qi = 0; qi < p.n_q; ++qi) {
-    float mmax = -CUDART_INF_F;
-    for (int s = 0; s < S; ++s) mmax = fmaxf(mmax, p.part_lse[(base + s) * kTokTile + qi]);
-    float wsum = 0.f;
-    float acc = 0.f;
-    if (mmax != -CUDART_INF_F) {
-      for (int s = 0; s < S; ++s) {
-        const float w = exp2f(p.part_lse[(base + s) * kTokTile + qi] - mmax);
-        wsum += w;
-        acc += w * p.part_o[((base + s) * kTokTile + qi) * kD + d];
-      }
-    }
-    const float o = wsum > 0.f ? acc / wsum : 0.f;
-    p.out[(static_cast<size_t>(b) * p.n_q + qi) * p.out_stride + h * kD + d] = __float2half_rn(o);
-    if (p.lse != nullptr && d == 0) {
-      p.lse[(static_cast<size_t>(b) * H + h) * p.n_q + qi] =
-          wsum > 0.f ? (mmax + log2f(wsum)) * 0.6931471805599453f : -CUDART_INF_F;
+  float mmax = -CUDART_INF_F;
+  for (int s = 0; s < S; ++s) mmax = fmaxf(mmax, p.part_lse[(base + s) * kTokTile + qi]);
+  float wsum = 0.f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (mmax != -CUDART_INF_F) {
+    for (int s = 0; s < S; ++s) {
+      const float w = exp2f(p.part_lse[(base + s) * kTokTile + qi] - mmax);
+      const float4 v = *reinterpret_cast<const float4*>(p.part_o + ((base + s) * kTokTile + qi) * kD + lane * 4);
+      wsum += w;
+      acc.x += w * v.x;
+      acc.y += w * v.y;
+      acc.z += w * v.z;
+      acc.w += w * v.w;
     }
   }
+  const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+  uint2 pk;
+  pk.x = pack_half2(acc.x * inv, acc.y * inv);
+  pk.y = pack_half2(acc.z * inv, acc.w * inv);
+  *reinterpret_cast<uint2*>(p.out + (static_cast<size_t>(b) * p.n_q + qi) * p.out_stride + h * kD + lane * 4) = pk;
+  if (p.lse != nullptr && lane == 0)
+    p.lse[(static_cast<size_t>(b) * H + h) * p.n_q + qi] =
+        wsum > 0.f ? (mmax + log2f(wsum)) * 0.6931471805599453f : -CUDART_INF_F;
 }
 
 }  // namespace
@@ -517,8 +524,8 @@ cudaError_t launch_attention(const AttnArgs& a_in, int B, int cache_dtype, cudaS
   }
   cudaError_t e = launch_ex(fn, grid, dim3(kThreads), smem, stream, pdl, kargs, 1, cm ? a.n_splits : 1);
   if (e != cudaSuccess || a.n_splits <= kMaxClusterSplits) return e;
-  return launch_ex(reinterpret_cast<const void*>(&attn_combine_kernel), dim3(a.n_heads, B), dim3(kD), 0, stream,
-                   pdl, kargs);
+  return launch_ex(reinterpret_cast<const void*>(&attn_combine_kernel), dim3(a.n_heads, B, (a.n_q + 7) / 8), dim3(256),
+                   0, stream, pdl, kargs);
 }
 
 }  // namespace fsx
