@@ -60,6 +60,18 @@ __host__ __device__ constexpr size_t attn_smem_bytes() {
 
 __device__ __forceinline__ int swz(int row, int unit) { return row * kUnits + (unit ^ (row & 7)); }
 
+// 2^x on the special-function unit (relative error about 2^-22; -inf -> +0)
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// The running maximum is only moved when a row's chunk maximum exceeds it by more
+// than this (log2 units), so P <= 2^8 stays well inside fp16 and the rescale of the
+// accumulators is skipped for most chunks; the result does not depend on it.
+constexpr float kLazyRescale = 8.f;
+
 // wait until at most n of this thread's cp.async groups are pending
 __device__ __forceinline__ void cp_async_wait_n(int n) {
   if (n <= 0) cp_async_wait<0>();
@@ -165,13 +177,39 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
     return;
   }
 
-  // ---- stage chunk c (keys kbeg + 64c ...) into raw stage s
+  // ---- stage chunk c (keys kbeg + kChunk c ...) into raw stage s
+  constexpr int UPR = RB / 16;               // 16-byte units per raw row
+  constexpr int RPP = kThreads / UPR;        // raw rows per pass of the CTA
+  constexpr int RAW_PASSES = (kChunk + RPP - 1) / RPP;
+  static_assert(kThreads % UPR == 0, "whole raw rows per pass");
+  const int su = tid % UPR;
+  const int sr = tid / UPR;
+  const size_t tok_bytes = static_cast<size_t>(H) * RB;  // bytes between two tokens of one head
+  const unsigned char* kbase =
+      reinterpret_cast<const unsigned char*>(kc) + (static_cast<size_t>(o_lo) * H + h) * RB + su * 16;
+  const unsigned char* vbase =
+      reinterpret_cast<const unsigned char*>(vc) + (static_cast<size_t>(o_lo) * H + h) * RB + su * 16;
   auto issue_chunk = [&](int c, int s) {
     const long long c0 = kbeg + static_cast<long long>(c) * kChunk;
     const int rows = static_cast<int>(min(static_cast<long long>(kChunk), kend - c0));
-    constexpr int UPR = RB / 16;  // 16-byte units per raw row
     unsigned char* kr = raw + (static_cast<size_t>(s) * 2 + 0) * kChunk * RB;
     unsigned char* vr = raw + (static_cast<size_t>(s) * 2 + 1) * kChunk * RB;
+    if (c0 + kChunk <= L) {  // cache rows only: fixed (row, unit) per thread
+      const size_t g = static_cast<size_t>(c0 + sr) * tok_bytes;
+      const unsigned char* ks = kbase + g;
+      const unsigned char* vs = vbase + g;
+      const uint32_t kd = smem_addr(kr + sr * RB + su * 16);
+      const uint32_t vd = smem_addr(vr + sr * RB + su * 16);
+#pragma unroll
+      for (int k = 0; k < RAW_PASSES; ++k) {
+        if (sr + k * RPP < rows) {
+          cp_async_16(kd + k * RPP * RB, ks + k * RPP * tok_bytes);
+          cp_async_16(vd + k * RPP * RB, vs + k * RPP * tok_bytes);
+        }
+      }
+      cp_async_commit();
+      return;
+    }
     for (int i = tid; i < rows * UPR; i += kThreads) {
       const int r = i / UPR;
       const int u = i - r * UPR;
@@ -237,7 +275,26 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
       const unsigned char* kr = raw + (static_cast<size_t>(s) * 2 + 0) * kChunk * RB;
       const unsigned char* vr = raw + (static_cast<size_t>(s) * 2 + 1) * kChunk * RB;
       constexpr int SRC_UNIT = RB / kUnits;  // raw bytes per 16-byte fp16 unit
-      for (int i = tid; i < kChunk * kUnits; i += kThreads) {
+      constexpr int TPP = kThreads / kUnits;  // tile rows per pass
+      static_assert(kThreads % kUnits == 0, "whole tile rows per pass");
+      if (c0 + kChunk <= L) {  // cache rows only
+        const int u = tid % kUnits;
+#pragma unroll
+        for (int k = 0; k < (kChunk + TPP - 1) / TPP; ++k) {
+          const int r = tid / kUnits + k * TPP;
+          if (r < kChunk) {
+            uint4* kd = kt + swz(r, u);
+            uint4* vd = vt + swz(r, u);
+            if (r < rows) {
+              convert_unit<CT>(kr + static_cast<size_t>(r) * RB + u * SRC_UNIT, kd, false);
+              convert_unit<CT>(vr + static_cast<size_t>(r) * RB + u * SRC_UNIT, vd, false);
+            } else {
+              *kd = make_uint4(0u, 0u, 0u, 0u);
+              *vd = make_uint4(0u, 0u, 0u, 0u);
+            }
+          }
+        }
+      } else for (int i = tid; i < kChunk * kUnits; i += kThreads) {
         const int r = i / kUnits;
         const int u = i - r * kUnits;
         uint4* kd = kt + swz(r, u);
@@ -272,16 +329,20 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
         mma_f16_16816(sc[j], qf[2 * dd + 1][0], qf[2 * dd + 1][1], qf[2 * dd + 1][2], qf[2 * dd + 1][3], b2, b3);
       }
     }
-    // ---- online softmax (log2 domain), masking keys past the range
+    // ---- online softmax (log2 domain; the 1/sqrt(d) log2(e) scale is applied inside
+    // the exponent), masking keys past the range on a ragged chunk only
+    if (rows < kChunk) {
+#pragma unroll
+      for (int j = 0; j < kNT; ++j) {
+        const int key = j * 8 + 2 * (lane & 3);
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          if (key + (e & 1) >= rows) sc[j][e] = -CUDART_INF_F;
+      }
+    }
     float mx[2] = {-CUDART_INF_F, -CUDART_INF_F};
 #pragma unroll
     for (int j = 0; j < kNT; ++j) {
-      const int key = j * 8 + 2 * (lane & 3);
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const bool valid = (key + (e & 1)) < rows;
-        sc[j][e] = valid ? sc[j][e] * scale_log2 : -CUDART_INF_F;
-      }
       mx[0] = fmaxf(mx[0], fmaxf(sc[j][0], sc[j][1]));
       mx[1] = fmaxf(mx[1], fmaxf(sc[j][2], sc[j][3]));
     }
@@ -289,21 +350,35 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
     for (int r = 0; r < 2; ++r) {
       mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
       mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
+      mx[r] *= scale_log2;
     }
-    float alpha[2], m_new[2], rs[2] = {0.f, 0.f};
+    if (__any_sync(0xffffffffu, mx[0] > m_run[0] + kLazyRescale || mx[1] > m_run[1] + kLazyRescale)) {
+      float alpha[2];
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      m_new[r] = fmaxf(m_run[r], mx[r]);
-      alpha[r] = exp2f(m_run[r] - m_new[r]);
-      m_run[r] = m_new[r];
+      for (int r = 0; r < 2; ++r) {
+        const float m_new = fmaxf(m_run[r], mx[r]);
+        alpha[r] = ex2_approx(m_run[r] - m_new);
+        m_run[r] = m_new;
+        l_run[r] *= alpha[r];
+      }
+#pragma unroll
+      for (int n = 0; n < 16; ++n) {
+        o_acc[n][0] *= alpha[0];
+        o_acc[n][1] *= alpha[0];
+        o_acc[n][2] *= alpha[1];
+        o_acc[n][3] *= alpha[1];
+      }
     }
+    const float nm0 = -m_run[0];
+    const float nm1 = -m_run[1];
+    float rs[2] = {0.f, 0.f};
     uint32_t pf[kKS][4];  // P as A fragments, one per k16 step of 16 keys
 #pragma unroll
     for (int j = 0; j < kNT; ++j) {
-      const float p0 = exp2f(sc[j][0] - m_new[0]);
-      const float p1 = exp2f(sc[j][1] - m_new[0]);
-      const float p2 = exp2f(sc[j][2] - m_new[1]);
-      const float p3 = exp2f(sc[j][3] - m_new[1]);
+      const float p0 = ex2_approx(fmaf(sc[j][0], scale_log2, nm0));
+      const float p1 = ex2_approx(fmaf(sc[j][1], scale_log2, nm0));
+      const float p2 = ex2_approx(fmaf(sc[j][2], scale_log2, nm1));
+      const float p3 = ex2_approx(fmaf(sc[j][3], scale_log2, nm1));
       rs[0] += p0 + p1;
       rs[1] += p2 + p3;
       const int kk = j >> 1;
@@ -319,14 +394,7 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
     for (int r = 0; r < 2; ++r) {
       rs[r] += __shfl_xor_sync(0xffffffffu, rs[r], 1);
       rs[r] += __shfl_xor_sync(0xffffffffu, rs[r], 2);
-      l_run[r] = l_run[r] * alpha[r] + rs[r];
-    }
-#pragma unroll
-    for (int n = 0; n < 16; ++n) {
-      o_acc[n][0] *= alpha[0];
-      o_acc[n][1] *= alpha[0];
-      o_acc[n][2] *= alpha[1];
-      o_acc[n][3] *= alpha[1];
+      l_run[r] += rs[r];
     }
     // ---- O += P V
 #pragma unroll
@@ -443,7 +511,6 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
   }
 }
 
-// Merge of the split partials of one (vehicle, head): 128 threads = 128 dims.
 // Merge of the split partials: one warp per (head, vehicle, query), lane = 4 dims; the
 // splits are added in split order.
 __global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs p) {
