@@ -5,11 +5,12 @@
 //
 // Split-KV flash decoding: the L_b + T keys of a vehicle are cut into
 // n_splits near-equal ranges; one CTA (3 warps x 16 queries = 48 query rows)
-// streams its range in 32-key chunks. Chunks are staged raw (bf16 / fp32 cache
-// rows, fp16 own rows) with 16-byte cp.async into a double buffer, converted
-// once to fp16 into an XOR-swizzled tile, and consumed by mma.sync m16n8k16
-// (S = Q K^T, then O += P V with P kept in registers) under an online softmax
-// in the log2 domain. With one split the CTA writes the normalised output.
+// streams its range in 32-key chunks. Each chunk is staged raw (bf16 / fp32 cache
+// rows, fp16 own rows) with 16-byte cp.async, converted once to fp16 into an
+// XOR-swizzled tile, and the next chunk is issued into the raw buffer while the
+// tile is consumed by mma.sync m16n8k16 (S = Q K^T with the query fragments read
+// from a shared tile, then O += P V with P kept in registers) under an online
+// softmax in the log2 domain. With one split the CTA writes the normalised output.
 // With 2..8 splits the splits of one (vehicle, head) form a thread-block
 // cluster: each CTA leaves (O / l, m + log2 l) in its shared memory and, after
 // a cluster barrier, merges a slice of the query rows over all splits through
@@ -35,10 +36,10 @@ constexpr int kThreads = kWarps * 32;
 #define FSX_ATTN_CHUNK 32
 #endif
 #ifndef FSX_ATTN_MIN_CTAS
-#define FSX_ATTN_MIN_CTAS 3
+#define FSX_ATTN_MIN_CTAS 5
 #endif
 #ifndef FSX_ATTN_RAW_STAGES
-#define FSX_ATTN_RAW_STAGES 2
+#define FSX_ATTN_RAW_STAGES 1
 #endif
 constexpr int kChunk = FSX_ATTN_CHUNK;  // keys per staged chunk
 constexpr int kRawStages = FSX_ATTN_RAW_STAGES;  // raw chunks staged (in flight while one is computed)
@@ -53,9 +54,14 @@ struct CacheRow {
 };
 
 // raw staging: [kRawStages][K|V][kChunk rows][row bytes]; compute tiles: fp16 [K|V][kChunk][kD] swizzled
+// The CTA's 48 query rows stay in shared memory and their fragments are re-read for
+// every chunk: that keeps the register budget at 128, so 5 CTAs (15 warps) share an SM.
+constexpr size_t kQTileBytes = static_cast<size_t>(kTokTile) * kD * 2;
+
 template <typename CT>
 __host__ __device__ constexpr size_t attn_smem_bytes() {
-  return static_cast<size_t>(kRawStages) * 2 * kChunk * CacheRow<CT>::kBytes + static_cast<size_t>(2) * kChunk * kD * 2;
+  return static_cast<size_t>(kRawStages) * 2 * kChunk * CacheRow<CT>::kBytes + static_cast<size_t>(2) * kChunk * kD * 2 +
+         kQTileBytes;
 }
 
 __device__ __forceinline__ int swz(int row, int unit) { return row * kUnits + (unit ^ (row & 7)); }
@@ -106,7 +112,7 @@ __device__ __forceinline__ void convert_unit<float>(const unsigned char* raw, ui
   }
 }
 
-static_assert((kTokTile + kMaxClusterSplits - 1) * (kD + 1) * 4 <= (2 * kRawStages + 2) * kChunk * kD * 2,
+static_assert((kTokTile + kMaxClusterSplits - 1) * (kD + 1) * 4 <= (2 * kRawStages + 2) * kChunk * kD * 2 + kQTileBytes,
               "the cluster merge buffers must fit in the staging memory");
 
 template <typename CT, bool CM>
@@ -235,20 +241,14 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
   // ---- Q fragments (A operand, 16 queries x 128) straight from global
   const int qr0 = warp * 16 + (lane >> 2);
   const int qr1 = qr0 + 8;
-  uint32_t qf[8][4];
-  {
-    const __half* q0 = p.q + (static_cast<size_t>(b) * p.n_q + qr0) * p.q_stride + h * kD;
-    const __half* q1 = p.q + (static_cast<size_t>(b) * p.n_q + qr1) * p.q_stride + h * kD;
-    const bool v0 = qr0 < p.n_q;
-    const bool v1 = qr1 < p.n_q;
-#pragma unroll
-    for (int kk = 0; kk < 8; ++kk) {
-      const int c = kk * 16 + 2 * (lane & 3);
-      qf[kk][0] = v0 ? *reinterpret_cast<const uint32_t*>(q0 + c) : 0u;
-      qf[kk][1] = v1 ? *reinterpret_cast<const uint32_t*>(q1 + c) : 0u;
-      qf[kk][2] = v0 ? *reinterpret_cast<const uint32_t*>(q0 + c + 8) : 0u;
-      qf[kk][3] = v1 ? *reinterpret_cast<const uint32_t*>(q1 + c + 8) : 0u;
-    }
+  uint4* qt = tile + 2 * kChunk * kUnits;  // [kTokTile][kD] fp16 queries, swizzled
+  for (int i = tid; i < kTokTile * kUnits; i += kThreads) {
+    const int r = i / kUnits;
+    const int u = i - r * kUnits;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (r < p.n_q)
+      v = *reinterpret_cast<const uint4*>(p.q + (static_cast<size_t>(b) * p.n_q + r) * p.q_stride + h * kD + u * 8);
+    qt[swz(r, u)] = v;  // made visible by the first chunk's barrier
   }
 
   float o_acc[16][4];
@@ -319,14 +319,22 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
     for (int j = 0; j < kNT; ++j) {
 #pragma unroll
       for (int e = 0; e < 4; ++e) sc[j][e] = 0.f;
+    }
 #pragma unroll
-      for (int dd = 0; dd < 4; ++dd) {  // 32 dims per ldmatrix.x4
+    for (int dd = 0; dd < 4; ++dd) {  // 32 dims per ldmatrix.x4
+      uint32_t qa[2][4];  // A fragments of the two 16-dim k steps
+      const int qrow = warp * 16 + (lane & 15);
+#pragma unroll
+      for (int t = 0; t < 2; ++t)
+        ldsm_x4(qa[t][0], qa[t][1], qa[t][2], qa[t][3], smem_addr(qt + swz(qrow, (2 * dd + t) * 2 + (lane >> 4))));
+#pragma unroll
+      for (int j = 0; j < kNT; ++j) {
         const int row = j * 8 + (lane & 7);
         const int unit = dd * 4 + (lane >> 3);
         uint32_t b0, b1, b2, b3;
         ldsm_x4(b0, b1, b2, b3, smem_addr(kt + swz(row, unit)));
-        mma_f16_16816(sc[j], qf[2 * dd][0], qf[2 * dd][1], qf[2 * dd][2], qf[2 * dd][3], b0, b1);
-        mma_f16_16816(sc[j], qf[2 * dd + 1][0], qf[2 * dd + 1][1], qf[2 * dd + 1][2], qf[2 * dd + 1][3], b2, b3);
+        mma_f16_16816(sc[j], qa[0][0], qa[0][1], qa[0][2], qa[0][3], b0, b1);
+        mma_f16_16816(sc[j], qa[1][0], qa[1][1], qa[1][2], qa[1][3], b2, b3);
       }
     }
     // ---- online softmax (log2 domain; the 1/sqrt(d) log2(e) scale is applied inside
