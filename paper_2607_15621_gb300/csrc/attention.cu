@@ -578,10 +578,11 @@ cudaError_t attention_set_attributes() {
     cudaError_t e = cudaFuncSetAttribute(fns[i], cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes[i]));
     if (e != cudaSuccess) return e;
   }
-  return cudaSuccess;
+  return attention_tc_set_attributes();
 }
 
 cudaError_t launch_attention(const AttnArgs& a_in, int B, int cache_dtype, cudaStream_t stream, bool pdl) {
+  if (attention_tc_eligible(a_in, cache_dtype)) return launch_attention_tc(a_in, B, stream, pdl);
   AttnArgs a = a_in;
   void* kargs[] = {&a};
   const dim3 grid(a.n_splits, a.n_heads, B);

@@ -56,6 +56,10 @@ struct AttnArgs {
 size_t attention_workspace_bytes(int B, int n_heads, int n_splits);
 cudaError_t launch_attention(const AttnArgs& a, int B, int cache_dtype, cudaStream_t stream, bool pdl);
 cudaError_t attention_set_attributes();
+// tcgen05 path: bf16 cache, one split, n_q <= 48, 1 <= n_own <= 64
+bool attention_tc_eligible(const AttnArgs& a, int cache_dtype);
+cudaError_t launch_attention_tc(const AttnArgs& a, int B, cudaStream_t stream, bool pdl);
+cudaError_t attention_tc_set_attributes();
 int attention_launch_count(int n_splits);
 
 // --------------------------------------------------------- embed / head
