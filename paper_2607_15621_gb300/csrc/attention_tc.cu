@@ -1,17 +1,19 @@
 // Eq. 1 of Sec. 3.1 on the 5th-generation tensor cores: one CTA per (vehicle,
 // head) computes softmax(Q [K_vlm ; K_ae]^T / sqrt(128)) [V_vlm ; V_ae] for the
 // expert's queries (at most 48, padded to an M = 64 tile) with a bf16 backbone
-// cache, one split. Q, K and V are fp16 with fp32 accumulation: the bf16 cache rows
-// are converted in shared memory (exact for |x| in [2^-14, 65504]) by the warps
-// that stage them. P is split into fp16 P_hi + P_lo (about 22 significant bits), so
-// P V carries almost no rounding of P.
+// cache, one split, fp32 accumulation. S = Q K^T in fp16: the bf16 cache K rows are
+// converted in shared memory (exact for |x| in [2^-14, 65504]) by the warps that
+// stage them. P V keeps the cache V rows in bf16 and splits P into bf16 P_hi + P_lo
+// (16 significant bits, more than fp16's 11); the own chunk (fp16 V) splits P into
+// fp16 P_hi + P_lo instead.
 //
 // Data path ("slot" = 64 keys; shared-memory operands 128-byte swizzled):
 //   Q             [64 q][128 d] fp16   smem, A of S          (K-major)
 //   K slot (x3)   [64 keys][128 d]     smem, B of S          (K-major)
-//   V slot (x3)   [64 keys][128 d]     smem, B of P V        (N = d contiguous, MN-major)
+//   V slot (x3)   [64 keys][128 d]     smem, B of P V        (N = d contiguous, MN-major;
+//                                      bf16 cache rows, fp16 own rows)
 //   S (x2)        [64 q][64 keys] fp32 tensor memory, 64 columns each
-//   P_hi, P_lo    [64 q][64 keys] fp16 tensor memory, A of P V, written over the
+//   P_hi, P_lo    [64 q][64 keys]      tensor memory, A of P V, written over the
 //                                      S buffer they were computed from (32 columns each)
 //   O             [64 q][128 d] fp32   tensor memory, 128 columns
 //   Row q of an M = 64 tile lives in lane (q mod 16) + 32 (q / 16).
@@ -19,8 +21,8 @@
 // [64 j, 64 j + 64); chunk i sits in K / V slot i mod 3.
 //
 // Warp roles (256 threads): warps 0-2 run the online softmax for query rows
-// 16 w + lane (lanes 0-15); warp 3 lane 0 issues S and P V as their inputs become
-// ready; warps 4-5 stage and convert the K rows, warps 6-7 the V rows, two chunks ahead.
+// 16 w .. 16 w + 15, two rows per thread; warp 3 lane 0 issues S and P V as their inputs become
+// ready; warps 4-5 stage (and convert) the K rows, warps 6-7 the V rows, two chunks ahead.
 // Every wait is bounded; a timeout raises the status word and the CTA drains its
 // MMAs before it frees the tensor memory.
 #include <math_constants.h>
@@ -88,6 +90,13 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+// two fp32 -> bf16x2 (round to nearest even), lo in the low half
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
 // D[tmem] (+)= A[tmem] * B[smem]^T, one K = 16 step (A: M rows in the D lane layout,
 // two 16-bit values per column)
 __device__ __forceinline__ void umma_f16_ta(uint32_t tmem_d, uint32_t tmem_a, uint64_t b_desc, uint32_t idesc,
@@ -138,28 +147,37 @@ __device__ __forceinline__ bool test_bar(uint64_t* bar, uint32_t parity) {
   return done != 0;
 }
 
-__device__ __forceinline__ void tmem_ld32_wait(uint32_t taddr, uint32_t (&r)[32]) {
-  tmem_ld32_issue(taddr, r);
+// 16 lanes x 256 bits, 8 repetitions along the columns: thread t gets, per 8-column
+// group g, lane t / 4 columns 8 g + 2 (t mod 4) + {0, 1}, then lane t / 4 + 8 the same
+__device__ __forceinline__ void tmem_ld_16x256b_x8(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x256b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
   tmem_wait_ld32(r);
 }
-
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+__device__ __forceinline__ void tmem_st_16x256b_x8(uint32_t taddr, const uint32_t (&r)[32]) {
   asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
-          taddr),
-      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
-      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
-      : "memory");
-}
-
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "tcgen05.st.sync.aligned.16x256b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
       "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
       "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
       "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]),
       "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]),
       "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+// 16 lanes x 128 bits, 8 repetitions: thread t gets, per 4-column group j, column
+// 4 j + (t mod 4) of lane t / 4, then of lane t / 4 + 8
+__device__ __forceinline__ void tmem_st_16x128b_x8(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x128b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
       : "memory");
 }
 
@@ -296,7 +314,8 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       const uint32_t id_s = idesc_f16_mn(64, kSlotKeys, false);
-      const uint32_t id_pv = idesc_f16_mn(64, kD, true);
+      const uint32_t id_pv_own = idesc_f16_mn(64, kD, true);       // fp16 P, fp16 own V
+      const uint32_t id_pv = idesc_f16_mn(64, kD, true) | (1u << 7) | (1u << 10);  // bf16 P, bf16 cache V
       const uint32_t aq = smem_addr(qt);
       auto issue_s = [&](int i) {  // S of chunk i into buffer i & 1
         const uint32_t d = tmem + kColS + (i & 1) * kSlotKeys;
@@ -312,11 +331,12 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
       auto issue_pv = [&](int i) {  // O (+)= P V of chunk i, P from tensor memory
         const uint32_t pa = tmem + kColS + (i & 1) * kSlotKeys;
         const uint32_t vb = smem_addr(vslot + (i % kSlots) * kSlotBytes);
+        const uint32_t idv = i == 0 ? id_pv_own : id_pv;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {  // 16 keys = 8 columns of packed fp16 pairs
           const uint64_t bd = sw128_desc_mn(vb + kk * 2048, 8192, 1024);
-          umma_f16_ta(tmem + kColO, pa + kk * 8, bd, id_pv, (i > 0 || kk > 0) ? 1u : 0u);  // P_hi
-          umma_f16_ta(tmem + kColO, pa + kSlotKeys / 2 + kk * 8, bd, id_pv, 1u);          // P_lo
+          umma_f16_ta(tmem + kColO, pa + kk * 8, bd, idv, (i > 0 || kk > 0) ? 1u : 0u);  // P_hi
+          umma_f16_ta(tmem + kColO, pa + kSlotKeys / 2 + kk * 8, bd, idv, 1u);          // P_lo
         }
         umma_commit(vempty + (i % kSlots));
         umma_commit(pvdone + (i & 1));
@@ -377,7 +397,7 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
         refilled = __all_sync(0xffffffffu, test_bar(empty + ((i + 2) % kSlots), ((i + 2) / kSlots) & 1));
         if (refilled) issue(i + 2);
       }
-      if (i > 0) {
+      if (i > 0 && !is_v) {  // cache K rows -> fp16 (V stays bf16)
         unsigned char* slot = pslots + (i % kSlots) * kSlotBytes;
 #pragma unroll 8
         for (int m = 0; m < kSlotKeys / 4; ++m) {
@@ -396,12 +416,19 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
     cp_async_wait<0>();
   } else {
     // ---------------------------------------------------------------- softmax rows
-    const int q = warp * 16 + lane;  // valid for lane < 16
-    const bool row_lane = lane < 16;
+    // Warp w owns query rows 16 w .. 16 w + 15 (tensor-memory lanes 32 w .. + 15).
+    // With the 16x256b load shape each thread holds rows ra = 16 w + t / 4 and
+    // rb = ra + 8, and the key pairs 8 g + 2 (t mod 4) + {0, 1} of every 8-key group
+    // g; a row's maximum and sum are completed across the 4 threads of a quad. Its
+    // P pairs are exactly the packed columns 4 g + (t mod 4) that the 16x128b store
+    // shape gives the same thread.
+    const int t4 = lane & 3;
+    const int ra = warp * 16 + (lane >> 2);
+    const int rbw = ra + 8;
     const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
     const float scale_log2 = 1.4426950408889634f * rsqrtf(static_cast<float>(kD));
-    float m_run = -CUDART_INF_F;
-    float l_run = 0.f;
+    float m_run[2] = {-CUDART_INF_F, -CUDART_INF_F};
+    float l_run[2] = {0.f, 0.f};
     bool ok = true;
     for (int i = 0; i < n_chunks; ++i) {
       const int valid = chunk_rows(i);
@@ -409,98 +436,122 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
       if (!ok) break;
       tc_fence_after();
       const uint32_t sbuf = tmem + lane_base + kColS + (i & 1) * kSlotKeys;
-      uint32_t sv[2][32];
-      tmem_ld32_issue(sbuf, sv[0]);
-      tmem_ld32_issue(sbuf + 32, sv[1]);
-      tmem_wait_ld32(sv[0]);
-      tmem_wait_ld32(sv[1]);
-      float s[64];
+      uint32_t sv[32];  // [g][row a: 2 keys, row b: 2 keys]
+      tmem_ld_16x256b_x8(sbuf, sv);
+      float s[2][16];   // [row][g * 2 + e] for key 8 g + 2 t4 + e
 #pragma unroll
-      for (int k = 0; k < 64; ++k) s[k] = __uint_as_float(sv[k >> 5][k & 31]);
+      for (int g = 0; g < 8; ++g)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          s[0][2 * g + e] = __uint_as_float(sv[4 * g + e]);
+          s[1][2 * g + e] = __uint_as_float(sv[4 * g + 2 + e]);
+        }
       if (valid < kSlotKeys) {
 #pragma unroll
-        for (int k = 0; k < 64; ++k)
-          if (k >= valid) s[k] = -CUDART_INF_F;
-      }
-      float mx = s[0];
+        for (int g = 0; g < 8; ++g)
 #pragma unroll
-      for (int k = 1; k < 64; ++k) mx = fmaxf(mx, s[k]);
-      mx *= scale_log2;
-      const bool grow = row_lane && mx > m_run + kLazyRescale;
+          for (int e = 0; e < 2; ++e)
+            if (8 * g + 2 * t4 + e >= valid) {
+              s[0][2 * g + e] = -CUDART_INF_F;
+              s[1][2 * g + e] = -CUDART_INF_F;
+            }
+      }
+      float mx[2], alpha[2] = {1.f, 1.f};
+      bool grow = false;
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        float m4[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) m4[e] = fmaxf(fmaxf(s[r][e], s[r][e + 4]), fmaxf(s[r][e + 8], s[r][e + 12]));
+        mx[r] = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+        mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
+        mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
+        mx[r] *= scale_log2;
+        grow = grow || mx[r] > m_run[r] + kLazyRescale;
+      }
       const bool any_grow = __any_sync(0xffffffffu, grow);
-      float alpha = 1.f;
       if (any_grow) {
-        const float m_new = grow ? mx : m_run;
-        alpha = ex2_approx(m_run - m_new);  // 0 for the first chunk
-        m_run = m_new;
-      }
-      const float nm = -m_run;
-      float rs = 0.f;
-      float pv[64];
 #pragma unroll
-      for (int k = 0; k < 64; ++k) {
-        pv[k] = ex2_approx(fmaf(s[k], scale_log2, nm));
-        rs += pv[k];
+        for (int r = 0; r < 2; ++r) {
+          const float m_new = fmaxf(m_run[r], mx[r]);
+          alpha[r] = ex2_approx(m_run[r] - m_new);  // 0 for the first chunk
+          m_run[r] = m_new;
+        }
       }
-      l_run = l_run * alpha + rs;
+      uint32_t ph[16], pl[16];  // 16x128b order: [g][row a, row b]
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const float nm = -m_run[r];
+        float r4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int g = 0; g < 8; ++g) {
+          const float p0 = ex2_approx(fmaf(s[r][2 * g], scale_log2, nm));
+          const float p1 = ex2_approx(fmaf(s[r][2 * g + 1], scale_log2, nm));
+          r4[g & 3] += p0 + p1;
+          uint32_t hi, lo;
+          if (i == 0) {  // own chunk: fp16 like its V rows
+            hi = pack_half2(p0, p1);
+            const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&hi));
+            lo = pack_half2(p0 - f.x, p1 - f.y);
+          } else {  // cache chunks: bf16 like the V rows
+            hi = pack_bf16x2(p0, p1);
+            lo = pack_bf16x2(p0 - __uint_as_float(hi << 16), p1 - __uint_as_float(hi & 0xffff0000u));
+          }
+          ph[2 * g + r] = hi;
+          pl[2 * g + r] = lo;
+        }
+        float rs = (r4[0] + r4[1]) + (r4[2] + r4[3]);
+        rs += __shfl_xor_sync(0xffffffffu, rs, 1);
+        rs += __shfl_xor_sync(0xffffffffu, rs, 2);
+        l_run[r] = l_run[r] * alpha[r] + rs;
+      }
       if (any_grow && i > 0) {
         // rescale this warp's O rows once P V of the previous chunk is done
         ok = wait_bar(pvdone + ((i - 1) & 1), ((i - 1) >> 1) & 1, p.status, abort);
         if (!ok) break;
         tc_fence_after();
 #pragma unroll 1
-        for (int c = 0; c < kD; c += 32) {
+        for (int c = 0; c < kD; c += 64) {
           uint32_t o[32];
-          tmem_ld32_wait(tmem + lane_base + kColO + c, o);
+          tmem_ld_16x256b_x8(tmem + lane_base + kColO + c, o);
 #pragma unroll
-          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-          tmem_st32(tmem + lane_base + kColO + c, o);
+          for (int g = 0; g < 8; ++g)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) o[4 * g + e] = __float_as_uint(__uint_as_float(o[4 * g + e]) * alpha[e >> 1]);
+          tmem_st_16x256b_x8(tmem + lane_base + kColO + c, o);
         }
       }
-      // P = P_hi + P_lo (fp16 each, about 22 significant bits) over the S it came from:
-      // P_hi in columns 0..31, P_lo in 32..63
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        uint32_t ph[16], pl[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          const float p0 = pv[hh * 32 + 2 * e];
-          const float p1 = pv[hh * 32 + 2 * e + 1];
-          ph[e] = pack_half2(p0, p1);
-          const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&ph[e]));
-          pl[e] = pack_half2(p0 - f.x, p1 - f.y);
-        }
-        tmem_st16(sbuf + hh * 16, ph);
-        tmem_st16(sbuf + kSlotKeys / 2 + hh * 16, pl);
-      }
+      // P = P_hi + P_lo over the S it came from: P_hi in columns 0..31, P_lo in 32..63
+      tmem_st_16x128b_x8(sbuf, ph);
+      tmem_st_16x128b_x8(sbuf + kSlotKeys / 2, pl);
       asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
       tc_fence_before();
       mbar_arrive(pfull + (i & 1));
     }
     if (ok && wait_bar(drain, 0, p.status, abort)) {  // every P V done
       tc_fence_after();
-      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-      const bool out_row = row_lane && q < p.n_q;
-      __half* orow = p.out + (static_cast<size_t>(b) * p.n_q + (out_row ? q : 0)) * p.out_stride + h * kD;
+      const float inv[2] = {l_run[0] > 0.f ? 1.f / l_run[0] : 0.f, l_run[1] > 0.f ? 1.f / l_run[1] : 0.f};
+      const bool va = ra < p.n_q;
+      const bool vb = rbw < p.n_q;
+      __half* oa = p.out + (static_cast<size_t>(b) * p.n_q + (va ? ra : 0)) * p.out_stride + h * kD + 2 * t4;
+      __half* ob = p.out + (static_cast<size_t>(b) * p.n_q + (vb ? rbw : 0)) * p.out_stride + h * kD + 2 * t4;
 #pragma unroll 1
-      for (int c = 0; c < kD; c += 32) {
+      for (int c = 0; c < kD; c += 64) {
         uint32_t o[32];
-        tmem_ld32_wait(tmem + lane_base + kColO + c, o);
-        if (out_row) {
+        tmem_ld_16x256b_x8(tmem + lane_base + kColO + c, o);
 #pragma unroll
-          for (int e = 0; e < 32; e += 8) {
-            uint4 w;
-            w.x = pack_half2(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv);
-            w.y = pack_half2(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
-            w.z = pack_half2(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv);
-            w.w = pack_half2(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv);
-            *reinterpret_cast<uint4*>(orow + c + e) = w;
-          }
+        for (int g = 0; g < 8; ++g) {
+          if (va) *reinterpret_cast<uint32_t*>(oa + c + 8 * g) =
+              pack_half2(__uint_as_float(o[4 * g]) * inv[0], __uint_as_float(o[4 * g + 1]) * inv[0]);
+          if (vb) *reinterpret_cast<uint32_t*>(ob + c + 8 * g) =
+              pack_half2(__uint_as_float(o[4 * g + 2]) * inv[1], __uint_as_float(o[4 * g + 3]) * inv[1]);
         }
       }
-      if (out_row && p.lse != nullptr)
-        p.lse[(static_cast<size_t>(b) * H + h) * p.n_q + q] =
-            l_run > 0.f ? (m_run + log2f(l_run)) * 0.6931471805599453f : -CUDART_INF_F;
+      if (p.lse != nullptr && t4 == 0) {
+        float* lrow = p.lse + (static_cast<size_t>(b) * H + h) * p.n_q;
+        if (va) lrow[ra] = l_run[0] > 0.f ? (m_run[0] + log2f(l_run[0])) * 0.6931471805599453f : -CUDART_INF_F;
+        if (vb) lrow[rbw] = l_run[1] > 0.f ? (m_run[1] + log2f(l_run[1])) * 0.6931471805599453f : -CUDART_INF_F;
+      }
     }
   }
 
