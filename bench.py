@@ -38,7 +38,7 @@ KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down", "persistent"]
 NCU_TRAFFIC = {
     ("persistent", "bf16_b1_l224"): 793.150976e6 + 3.595776e6,   # persistent_tick_bf16_b1_l224.md
     ("qkv", "bf16_b128_ragged"): 18.229504e6 + 71.913728e6,      # gemm_tc_bf16_b128_ragged.md
-    ("attention", "bf16_b128_ragged"): 2262.161e6 + 45.69216e6,  # attn_splitkv_bf16_b128_ragged.md
+    ("attention", "bf16_b128_ragged"): 2258.334e6 + 39.689472e6,  # attn_tc_bf16_b128_ragged.md
 }
 
 
