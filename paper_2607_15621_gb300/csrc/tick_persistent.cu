@@ -63,6 +63,9 @@ constexpr int kActAtom = kTokTile * 128;      // one K slice of the 48 token row
 constexpr uint32_t kTmemCols = 64;            // accumulator: 128 lanes x 48 fp32 columns
 constexpr uint32_t kIdesc = idesc_f16(128, kTokTile);
 constexpr unsigned long long kSpinLimitNs = 1000000000ull;
+#ifndef FSX_NORM_SPLIT
+#define FSX_NORM_SPLIT 1
+#endif
 #ifndef FSX_NORM_BATCH
 #define FSX_NORM_BATCH 2
 #endif
@@ -360,6 +363,45 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     __syncthreads();
   };
 
+  // RMSNorm split along K inside the cluster (phase A): this rank reads only its 128
+  // columns of x, sends its per-token partial sums of x^2 to every rank, normalises its
+  // columns and writes them into the activation image of all four ranks, so each CTA
+  // holds the full [48 x 512] fp16 image for its QKV rows. gss lives in dstT, idle
+  // from the end of the previous phase B to the W_o transpose.
+  auto load_normalized_split = [&](const float* Xs) {
+    float* gss = dstT;  // [4 ranks][48]
+    constexpr int kRowsPerWarp = kTokTile / (kThr / 32);  // 6
+    float4 xv[kRowsPerWarp];
+#pragma unroll
+    for (int i = 0; i < kRowsPerWarp; ++i) {
+      const int r = warp + 8 * i;
+      xv[i] = r < T ? ld_cg4(Xs + static_cast<size_t>(r) * d + rank * 128 + lane * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int i = 0; i < kRowsPerWarp; ++i) {
+      const int r = warp + 8 * i;
+      const float ps = warp_sum(xv[i].x * xv[i].x + xv[i].y * xv[i].y + xv[i].z * xv[i].z + xv[i].w * xv[i].w);
+      if (r < T && lane < kCl) st_cluster_f32(cluster_addr(gss + rank * kTokTile + r, lane), ps);
+    }
+    cluster.sync();  // every rank's partial sums arrived
+#pragma unroll
+    for (int i = 0; i < kRowsPerWarp; ++i) {
+      const int r = warp + 8 * i;
+      if (r < T) {
+        const float ss = ((gss[r] + gss[kTokTile + r]) + gss[2 * kTokTile + r]) + gss[3 * kTokTile + r];
+        const float rstd = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
+        const float lo = __uint_as_float(pack_half2(xv[i].x * rstd, xv[i].y * rstd));
+        const float hi = __uint_as_float(pack_half2(xv[i].z * rstd, xv[i].w * rstd));
+        unsigned char* dst = act + sw128_offset(kTokTile, r, rank * 128 + lane * 4);
+#pragma unroll
+        for (int peer = 0; peer < kCl; ++peer) st_cluster_v2f(cluster_addr(dst, peer), lo, hi);
+      }
+    }
+    asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+    cluster.sync();  // the full image is in every rank
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // visible to the tensor core
+  };
+
   // add the CTA's [48 x 128] transposed output (dstT) into X_next columns col0..col0+127,
   // plus the residual X_cur when this is cluster 0
   auto scatter_add = [&](float* Xn, const float* Xc, int col0, bool add_residual) {
@@ -505,7 +547,11 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       const int e1 = static_cast<int>(static_cast<long long>(n_elem) * (cta + 1) / G);
       for (int e = e0 + tid; e < e1; e += kThr) __stcg(Xz + e, 0.f);
     }
+#if FSX_NORM_SPLIT
+    load_normalized_split(Xc);
+#else
     load_normalized(Xc);
+#endif
 
     // --- QKV: D[96 (+32 unused) rows x 48 tokens] over K = 512; the 12 KB K
     // slices lie back to back in slots 0-5, so slice a needs the slots it touches
