@@ -30,13 +30,16 @@ sys.path.insert(0, ROOT)
 METRIC = "vehicle-ticks/s (1e6 / us-per-tick x B) of the action-expert tick"
 UNIT = "vehicle-ticks/s"
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_TENSOR_TFS = 1700.0      # dense bf16 / fp16, sustained (one earlier GB300 measurement)
+NOMINAL_HBM_GBS = 8000.0          # the HBM3e figure the tick roofline is stated against
+NOMINAL_TENSOR_TFS = 2250.0       # dense bf16 / fp16 tensor peak, nominal
 KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down", "persistent"]
 
 # DRAM bytes (read + write) of one launch of the timed kernel, from one ncu capture of the
 # kernel as it is now (profiles/ holds each summary with its command). A kernel that changed
 # after its capture gets no entry, so its traffic is reported as null.
 NCU_TRAFFIC = {
-    ("persistent", "bf16_b1_l224"): 793.150976e6 + 3.595776e6,   # persistent_tick_bf16_b1_l224.md
+    # the persistent tick changed after its last capture: no entry until it is captured again
     ("qkv", "bf16_b128_ragged"): 18.229504e6 + 71.913728e6,      # gemm_tc_bf16_b128_ragged.md
     ("attention", "bf16_b128_ragged"): 2258.334e6 + 39.689472e6,  # attn_tc_bf16_b128_ragged.md
 }
@@ -79,13 +82,16 @@ def max_over_ranks(value: float, device=None) -> float:
 
 
 def peaks():
+    """HBM copy GB/s and sustained dense bf16 TF/s of this GPU (fp16 runs at the bf16 rate)."""
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
         with open(path) as fh:
             p = json.load(fh)
-        return float(p["hbm_gbs"]), "measured"
+        hbm = float(p["hbm_gbs"])
     except Exception:
-        return FALLBACK_HBM_GBS, "fallback"
+        return FALLBACK_HBM_GBS, FALLBACK_TENSOR_TFS, "fallback"
+    tfs = p.get("bf16_tflops_sustained", p.get("bf16_tflops"))
+    return hbm, float(tfs) if tfs else FALLBACK_TENSOR_TFS, "measured"
 
 
 def workload_info(name):
@@ -100,6 +106,18 @@ def algorithmic_bytes(dims, lengths, cache_dtype, weight_bytes):
     elem = 2 if cache_dtype == "bf16" else 4
     kv = int(np.sum(lengths)) * dims.n_layers * 2 * dims.hd * elem
     return weight_bytes + kv, kv
+
+
+def tick_flops(dims, lengths):
+    """Per tick: the projection GEMMs (2 flop per weight per token) of every layer plus
+    Eq. 1 (Q K^T and P V over the cache and own keys: 4 T D flop per key, head and layer)."""
+    T, d, hd, f = dims.n_tok, dims.d_model, dims.hd, dims.d_ff
+    B = len(lengths)
+    per_layer_w = 3 * hd * d + d * hd + 2 * f * d + d * f
+    gemm = 2 * B * T * per_layer_w * dims.n_layers
+    keys = int(np.sum(lengths)) + B * T
+    attn = 4 * T * dims.head_dim * dims.n_heads * keys * dims.n_layers
+    return gemm + attn
 
 
 def start_clock_sampler(path, index):
@@ -290,10 +308,14 @@ def main():
     }[kclass]
     if unit_bytes is None:  # one launch = the whole tick: weights + cache rows
         unit_bytes = algorithmic_bytes(dims, lengths, dtype, ex.weight_bytes())[0]
-    hbm, peak_kind = peaks()
+    hbm, tensor_tfs, peak_kind = peaks()
     achieved = unit_bytes / per_launch_s / 1e9
     tick_bytes, kv_bytes = algorithmic_bytes(dims, lengths, dtype, ex.weight_bytes())
     tick_gbs = tick_bytes / (ms_per_step / 1e3) / 1e9
+    flops = tick_flops(dims, lengths)
+    # roofline time of one tick = max(bytes / HBM bandwidth, FLOPs / tensor peak)
+    rl_meas_us = max(tick_bytes / (hbm * 1e9), flops / (tensor_tfs * 1e12)) * 1e6
+    rl_nom_us = max(tick_bytes / (NOMINAL_HBM_GBS * 1e9), flops / (NOMINAL_TENSOR_TFS * 1e12)) * 1e6
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -309,7 +331,12 @@ def main():
                      "frac": achieved / hbm, "traffic": NCU_TRAFFIC.get((kclass, args.workload)), "peak_source": peak_kind,
                      "bytes_per_launch": unit_bytes, "launch_us": per_launch_s * 1e6},
         "tick_roofline": {"bytes_per_tick": tick_bytes, "kv_bytes_per_tick": kv_bytes, "achieved_gbs": tick_gbs,
-                          "frac_of_measured_hbm": tick_gbs / hbm, "frac_of_8tbs": tick_gbs / 8000.0},
+                          "frac_of_measured_hbm": tick_gbs / hbm, "frac_of_8tbs": tick_gbs / NOMINAL_HBM_GBS,
+                          "flops_per_tick": flops,
+                          "bound": "hbm" if tick_bytes / hbm >= flops / (tensor_tfs * 1e3) else "tensor",
+                          "roofline_us_measured_peaks": rl_meas_us, "frac_measured_peaks": rl_meas_us / (ms_per_step * 1e3),
+                          "roofline_us_8tbs_2250tf": rl_nom_us, "frac_8tbs_2250tf": rl_nom_us / (ms_per_step * 1e3),
+                          "peaks": {"hbm_gbs": hbm, "tensor_tflops_sustained": tensor_tfs, "source": peak_kind}},
         "e2e": {"value": world * B * e2e_steps / e2e_s, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h)},
         "clocks": clocks,

@@ -5,11 +5,13 @@
 // attention head (H clusters, 4H CTAs, one CTA per SM, all co-resident).
 // Every layer runs two phases separated by device-wide counters:
 //   phase A (every cluster = one head h):
-//     x -> RMSNorm (every CTA normalises all token rows itself, straight from
-//     L2) -> the CTA's 96 rows of [W_q; W_k; W_v] for head h (32 q, 32 k, 32 v
-//     dims) on the tensor cores (tcgen05, accumulator in tensor memory) ->
+//     x -> RMSNorm (split along K: each CTA normalises its 128 columns and
+//     sends them to the whole cluster) -> the CTA's 96 rows of
+//     [W_q; W_k; W_v] for head h (32 q, 32 k, 32 v dims) on the tensor cores
+//     (tcgen05, accumulator in tensor memory) ->
 //     q, k_ae, v_ae pushed to all 4 CTAs -> Eq. 1 over a quarter of
-//     [K_vlm ; K_ae] per CTA -> the 4 fp32 split results merged in shared memory
+//     [K_vlm ; K_ae] per CTA (cache rows staged three 64-key chunks deep in the
+//     shared memory the QKV operands used) -> the 4 fp32 split results merged
 //     (log-sum-exp weights) -> the CTA's 128 output columns of o_h W_o^T
 //     (tcgen05) added into the next residual state with vector atomics
 //     (cluster 0 also adds the residual itself).
@@ -27,13 +29,13 @@
 // order it consumes them, as the swizzled K-major images the tensor core reads
 // (128-byte swizzle, one 64-wide K slice per image), and streamed by bulk
 // copies through a 6-slot ring of 16 KB that is refilled as soon as a GEMM has
-// finished with its slots, so the HBM stream runs ahead across phases and
+// finished with its slots (slots 2-5 only once the attention has finished
+// staging cache rows in them), so the HBM stream runs ahead across phases and
 // layers. A layer takes 12 ring positions (6 of QKV, 2 of W_o, 2 of gate/up,
 // 1 of W_d and one empty position; CTAs without SwiGLU work leave positions
 // 8-11 empty), so the QKV images of every layer start at slot 0. The MMAs run
 // with M = 128: the 96-row QKV images are padded with whatever follows them in
-// shared memory, and the accumulator rows that produces are never read. The layer's backbone cache rows are prefetched into L2 at the start of
-// the layer and converted bf16/fp32 -> fp16 while staging 32-key tiles.
+// shared memory, and the accumulator rows that produces are never read.
 #include <cooperative_groups.h>
 #include <math_constants.h>
 
@@ -99,10 +101,6 @@ __device__ __forceinline__ void red_add_v4(float* addr, float4 v) {
   asm volatile("red.relaxed.gpu.global.add.v4.f32 [%0], {%1,%2,%3,%4};" ::"l"(addr), "f"(v.x), "f"(v.y), "f"(v.z),
                "f"(v.w)
                : "memory");
-}
-
-__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
 // Device-wide arrival counter: after the CTA barrier one thread adds 1 with
@@ -444,75 +442,108 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
                (first && kk == 0) ? 0u : 1u);
   };
 
-  // ---- this CTA's cache rows of a layer, staged in the activation image (free
-  // from the end of the QKV MMA to the next RMSNorm): two halves of kStageKeys
-  // keys, K rows then V rows, each row padded to kRowStride bytes so ldmatrix
-  // reads are conflict-free. Rows arrive raw (bf16 / fp32) by 16-byte cp.async
-  // copies spread over all threads and are converted to fp16 in place (at the
-  // start of the row).
+  // ---- this CTA's cache rows of a layer, staged in the shared memory that is idle
+  // from the end of the QKV MMA to the end of the attention: ring slots 2-5 and
+  // the activation image behind them (112 KB, contiguous). It is cut into kNB
+  // buffers of kStageKeys keys (K rows then V rows, each row padded to kRowStride
+  // bytes so ldmatrix reads are conflict-free), so kNB - 1 chunks are in flight
+  // while one is consumed. Rows arrive raw (bf16 / fp32) by 16-byte cp.async
+  // copies and are converted to fp16 in place (at the start of the row). Thread
+  // t always handles 16-byte units t, t + 256, ... of a buffer (row = unit >> s,
+  // no division), and the weight copies of positions 8-11 of the layer (slots
+  // 2-5) are issued only once the attention is done with the region.
   constexpr int kRowStride = sizeof(CT) == 2 ? kD * 2 + 16 : kD * 4 + 16;  // 272 / 528 bytes
-  constexpr int kHalfBytes = 8 * kActAtom / 2;                            // 24 KB (d = 512)
-  constexpr int kStageKeys = kHalfBytes / (2 * kRowStride);               // 45 / 23 keys
+  constexpr int kNB = 3;                                                  // staging buffers
+  constexpr int kStageRegion = 4 * kSlotBytes + 8 * kActAtom;             // 112 KB (d = 512)
+  constexpr int kStageKeys = sizeof(CT) == 2 ? 64 : 36;                   // two whole key tiles (bf16)
+  constexpr int kBufBytes = 2 * kStageKeys * kRowStride;                  // 34 / 37.1 KB
+  constexpr int kUnitsPerRow = kD * static_cast<int>(sizeof(CT)) / 16;   // raw 16-byte units: 16 / 32
+  constexpr int kUnitShift = sizeof(CT) == 2 ? 4 : 5;
+  constexpr int kRawIters = (2 * kStageKeys * kUnitsPerRow + kThr - 1) / kThr;  // 8 / 9
+  constexpr int kCvtIters = (2 * kStageKeys * 16 + kThr - 1) / kThr;            // fp16 units: 8 / 5
+  static_assert(kSlots == 6 && kPersistAChunks == 8, "staging assumes slots 2-5 hold positions 8-11");
+  static_assert((1 << kUnitShift) == kUnitsPerRow, "unit shift");
+  static_assert(kBufBytes % 16 == 0 && (kStageKeys * kRowStride) % 16 == 0, "cp.async / ldmatrix alignment");
+  static_assert(kNB * kBufBytes <= kStageRegion, "staging buffers exceed slots 2-5 + the activation image");
+  static_assert(sizeof(CT) == 4 || kStageKeys % (2 * kKeyTile) == 0, "an even number of key tiles per bf16 chunk");
+  static_assert(3 * 2 * 8 * 32 * 16 + 3 * 2 * 32 * 16 <= 8 * kActAtom, "key-half merge scratch exceeds the activation image");
+  unsigned char* const stage_base = ring + 2 * kSlotBytes;  // the activation image follows the ring
   const long long c_hi = min(kend, Lc);
   const int n_cache = c_hi > kbeg ? static_cast<int>(c_hi - kbeg) : 0;  // cache keys of this CTA
   const int n_chunks = (n_cache + kStageKeys - 1) / kStageKeys;
   const int own_lo = static_cast<int>(max(kbeg, Lc) - Lc);              // own keys of this CTA
   const int own_n = static_cast<int>(kend - Lc) - own_lo;
-  // all threads: 16-byte cp.async copies of chunk j into half j & 1 (one commit group)
-  constexpr int kUnitsPerRow = kD * static_cast<int>(sizeof(CT)) / 16;  // 16 / 32
-  auto stage_issue = [&](int j, const CT* kc, const CT* vc) {
+  const size_t tok_bytes = static_cast<size_t>(p.H) * kD * sizeof(CT);  // one token row of all heads
+  const size_t head_off = (static_cast<size_t>(o_lo + kbeg) * p.H + head) * kD * sizeof(CT);
+  // all threads: 16-byte cp.async copies of chunk j into buffer j % kNB (one commit group)
+  auto stage_issue = [&](int j, const unsigned char* kh, const unsigned char* vh) {
     const int k0 = j * kStageKeys;
     const int n = min(kStageKeys, n_cache - k0);
-    unsigned char* kb = act + (j & 1) * kHalfBytes;
-    for (int i = tid; i < 2 * n * kUnitsPerRow; i += kThr) {  // (K|V, key, unit)
-      const int kv = i / (n * kUnitsPerRow);
-      const int rest = i - kv * n * kUnitsPerRow;
-      const int key = rest / kUnitsPerRow;
-      const int u = rest - key * kUnitsPerRow;
-      const unsigned char* src = reinterpret_cast<const unsigned char*>(kv ? vc : kc) +
-                                 ((static_cast<size_t>(o_lo + kbeg + k0 + key) * p.H + head) * kD) * sizeof(CT) + u * 16;
-      cp_async_16(smem_addr(kb + kv * kStageKeys * kRowStride + key * kRowStride + u * 16), src);
+    unsigned char* kb = stage_base + (j % kNB) * kBufBytes;
+#pragma unroll
+    for (int it = 0; it < kRawIters; ++it) {
+      const int i = tid + it * kThr;
+      const int r = i >> kUnitShift;  // row of [K rows ; V rows]
+      const int u = i & (kUnitsPerRow - 1);
+      const bool is_v = r >= kStageKeys;
+      const int key = is_v ? r - kStageKeys : r;
+      if (r < 2 * kStageKeys && key < n)
+        cp_async_16(smem_addr(kb + r * kRowStride + u * 16),
+                    (is_v ? vh : kh) + static_cast<size_t>(k0 + key) * tok_bytes + u * 16);
     }
     cp_async_commit();
   };
   // all threads: wait for chunk j and convert it to fp16 in place
   auto stage_ready = [&](int j) {
-    const int h = j & 1;
-    if (j + 1 < n_chunks)  // chunk j + 1 is the only younger group in flight
+    const int younger = min(n_chunks - 1 - j, kNB - 1);  // groups of later chunks still in flight
+    if (younger >= 2)
+      cp_async_wait<2>();
+    else if (younger == 1)
       cp_async_wait<1>();
     else
       cp_async_wait<0>();
     __syncthreads();
     const int n = min(kStageKeys, n_cache - j * kStageKeys);
-    unsigned char* kb = act + h * kHalfBytes;
+    unsigned char* kb = stage_base + (j % kNB) * kBufBytes;
     if (sizeof(CT) == 2) {
-      for (int i = tid; i < 2 * n * 16; i += kThr) {  // (K|V, key, 16-byte unit)
-        const int kv = i / (n * 16);
-        const int rest = i - kv * n * 16;
-        uint4* ptr = reinterpret_cast<uint4*>(kb + kv * kStageKeys * kRowStride + (rest >> 4) * kRowStride + (rest & 15) * 16);
-        const uint4 raw = *ptr;
-        *ptr = make_uint4(bf16x2_to_half2(raw.x), bf16x2_to_half2(raw.y), bf16x2_to_half2(raw.z), bf16x2_to_half2(raw.w));
+      uint4 v[kCvtIters];
+#pragma unroll
+      for (int it = 0; it < kCvtIters; ++it) {  // every load before the first store
+        const int i = tid + it * kThr;
+        const int r = i >> 4;
+        const int key = r >= kStageKeys ? r - kStageKeys : r;
+        if (r < 2 * kStageKeys && key < n) v[it] = *reinterpret_cast<const uint4*>(kb + r * kRowStride + (i & 15) * 16);
+      }
+#pragma unroll
+      for (int it = 0; it < kCvtIters; ++it) {
+        const int i = tid + it * kThr;
+        const int r = i >> 4;
+        const int key = r >= kStageKeys ? r - kStageKeys : r;
+        if (r < 2 * kStageKeys && key < n)
+          *reinterpret_cast<uint4*>(kb + r * kRowStride + (i & 15) * 16) =
+              make_uint4(bf16x2_to_half2(v[it].x), bf16x2_to_half2(v[it].y), bf16x2_to_half2(v[it].z),
+                         bf16x2_to_half2(v[it].w));
       }
     } else {
-      // 32-byte fp32 unit u of a row -> 16-byte fp16 unit u at the row start: all reads
-      // of a round land before its writes, and a unit's input is never written by a
-      // later round
-      for (int base = 0; base < 2 * n * 16; base += kThr) {
-        const int i = base + tid;
+      // 32-byte fp32 unit u of a row -> 16-byte fp16 unit u at the row start. A row's 16
+      // units fall in one round of 256, all reads of a round land before its writes, and
+      // a unit's input is never written by a later round.
+#pragma unroll 1
+      for (int it = 0; it < kCvtIters; ++it) {
+        const int i = tid + it * kThr;
+        const int r = i >> 4;
+        const int key = r >= kStageKeys ? r - kStageKeys : r;
+        const bool live = r < 2 * kStageKeys && key < n;
+        unsigned char* row = kb + r * kRowStride;
+        const int u = i & 15;
         uint4 o = make_uint4(0u, 0u, 0u, 0u);
-        unsigned char* row = nullptr;
-        int u = 0;
-        if (i < 2 * n * 16) {
-          const int kv = i / (n * 16);
-          const int rest = i - kv * n * 16;
-          row = kb + kv * kStageKeys * kRowStride + (rest >> 4) * kRowStride;
-          u = rest & 15;
+        if (live) {
           const float4 a = *reinterpret_cast<const float4*>(row + u * 32);
           const float4 b = *reinterpret_cast<const float4*>(row + u * 32 + 16);
           o = make_uint4(pack_half2(a.x, a.y), pack_half2(a.z, a.w), pack_half2(b.x, b.y), pack_half2(b.z, b.w));
         }
         __syncthreads();
-        if (row != nullptr) *reinterpret_cast<uint4*>(row + u * 16) = o;
+        if (live) *reinterpret_cast<uint4*>(row + u * 16) = o;
         __syncthreads();
       }
     }
@@ -527,17 +558,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     float* Xc = X0 + static_cast<size_t>(sA % 3) * xs;        // layer input
     float* Xm = X0 + static_cast<size_t>((sA + 1) % 3) * xs;  // after attention
     float* Xz = X0 + static_cast<size_t>((sA + 2) % 3) * xs;  // zeroed now, written by phase B
-    const CT* kc = static_cast<const CT*>(p.targs->k_cache[layer]);
-    const CT* vc = static_cast<const CT*>(p.targs->v_cache[layer]);
-
-    // L2 prefetch of this layer's cache: CTA c takes whole token rows (all heads,
-    // contiguous) t = c, c + G, ..., spread over its threads, so the grid issues a
-    // handful of large prefetches instead of one per (token, head) row
-    for (long long t = cta + static_cast<long long>(G) * tid; t < Lc; t += static_cast<long long>(G) * kThr) {
-      const size_t row = static_cast<size_t>(o_lo + t) * p.H * kD;
-      prefetch_l2(kc + row, static_cast<uint32_t>(p.H * kD * sizeof(CT)));
-      prefetch_l2(vc + row, static_cast<uint32_t>(p.H * kD * sizeof(CT)));
-    }
+    // this CTA's first cache row (head h, key kbeg of the vehicle) in layer l's K and V
+    const unsigned char* kc = n_chunks > 0 ? static_cast<const unsigned char*>(p.targs->k_cache[layer]) + head_off : nullptr;
+    const unsigned char* vc = n_chunks > 0 ? static_cast<const unsigned char*>(p.targs->v_cache[layer]) + head_off : nullptr;
 
     // =========================== phase A ===========================
     wait_counter(p.counters + sA, sA == 0 ? G : n_b_ctas, p.status, abort);
@@ -569,7 +592,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       __syncwarp();
     }
     wait_mma();
-    for (int j = 0; j < 2 && j < n_chunks; ++j)  // the activation image is free: stage the cache rows
+    for (int j = 0; j < kNB && j < n_chunks; ++j)  // slots 2-5 and the activation image are free
       stage_issue(j, kc, vc);
     // rows 32j..32j+31 of the accumulator are q, k, v dims 32 rank .. 32 rank + 31
     if ((warp & 3) < 3) {
@@ -587,8 +610,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     }
     tc_fence_before();
     __syncthreads();
-    if (tid == 0)  // slots 0-5 are free: W_o, gate/up, W_d of this layer
-      for (int i = kSlots; i < kLayerChunks; ++i) issue(q0 + i);
+    if (tid == 0)  // slots 0, 1 are free: W_o of this layer (slots 2-5 stage the cache)
+      for (int i = kSlots; i < kPersistAChunks; ++i) issue(q0 + i);
     // this rank's 32 dims of q, k_ae, v_ae (48 rows x 64 bytes each) to the partners
     push_rows(qbuf + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
     push_rows(ownk + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
@@ -596,17 +619,18 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     cluster.sync();  // q, own k, own v complete in every CTA
 
     // --- Eq. 1 over keys [kbeg, kend) of [cache ; own] in 32-key tiles. Warp w < 6
-    // takes query rows 16 (w % 3) .. +15 and value dims 64 (w / 3) .. +63; both
-    // warps of a query tile compute the full scores, so no in-CTA merge is needed.
+    // takes query rows 16 (w % 3) .. +15 and every other key tile (tiles kh, kh + 2, ...
+    // of a chunk, kh = w / 3) over all 128 value dims; the two key halves of a query
+    // tile are merged in shared memory afterwards (log-sum-exp weights).
     const int qt = warp % 3;
-    const int dh = warp / 3;
-    float o_acc[8][4];
+    const int kh = warp / 3;
+    float o_acc[16][4];
     float m_run[2] = {-CUDART_INF_F, -CUDART_INF_F};
     float l_run[2] = {0.f, 0.f};
 #pragma unroll
-    for (int n = 0; n < 8; ++n)
+    for (int nb = 0; nb < 16; ++nb)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) o_acc[n][e] = 0.f;
+      for (int e = 0; e < 4; ++e) o_acc[nb][e] = 0.f;
     uint32_t qf[8][4];
     if (warp < 6) {
 #pragma unroll
@@ -615,9 +639,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         ldsm_x4(qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3], smem_addr(src));
       }
     }
-    // keys 0..n-1 with K rows at kb and V rows at vb (fp16, `stride` bytes apart)
+    // this warp's key tiles of keys 0..n-1, K rows at kb and V rows at vb (fp16, `stride` bytes apart)
     auto attend = [&](const unsigned char* kb, const unsigned char* vb, int stride, int n) {
-      for (int t0 = 0; t0 < n; t0 += kKeyTile) {
+      for (int t0 = kh * kKeyTile; t0 < n; t0 += 2 * kKeyTile) {
         const int rows = min(kKeyTile, n - t0);
         float sc[4][4];
 #pragma unroll
@@ -672,11 +696,11 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
           l_run[r] = l_run[r] * alpha[r] + rs[r];
         }
 #pragma unroll
-        for (int n = 0; n < 8; ++n) {
-          o_acc[n][0] *= alpha[0];
-          o_acc[n][1] *= alpha[0];
-          o_acc[n][2] *= alpha[1];
-          o_acc[n][3] *= alpha[1];
+        for (int nb = 0; nb < 16; ++nb) {
+          o_acc[nb][0] *= alpha[0];
+          o_acc[nb][1] *= alpha[0];
+          o_acc[nb][2] *= alpha[1];
+          o_acc[nb][3] *= alpha[1];
         }
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
@@ -684,9 +708,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
           r = r < n ? r : 0;
           const uint32_t vrow = smem_addr(vb + r * stride);
 #pragma unroll
-          for (int np = 0; np < 4; ++np) {
+          for (int np = 0; np < 8; ++np) {
             uint32_t b0, b1, b2, b3;
-            ldsm_x4_trans(b0, b1, b2, b3, vrow + (dh * 8 + np * 2 + (lane >> 4)) * 16);
+            ldsm_x4_trans(b0, b1, b2, b3, vrow + (np * 2 + (lane >> 4)) * 16);
             mma_f16_16816(o_acc[2 * np], pf[kk][0], pf[kk][1], pf[kk][2], pf[kk][3], b0, b1);
             mma_f16_16816(o_acc[2 * np + 1], pf[kk][0], pf[kk][1], pf[kk][2], pf[kk][3], b2, b3);
           }
@@ -696,15 +720,62 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     for (int j = 0; j < n_chunks; ++j) {
       stage_ready(j);
       if (warp < 6) {
-        const unsigned char* kb = act + (j & 1) * kHalfBytes;
+        const unsigned char* kb = stage_base + (j % kNB) * kBufBytes;
         attend(kb, kb + kStageKeys * kRowStride, kRowStride, min(kStageKeys, n_cache - j * kStageKeys));
       }
-      __syncthreads();  // half j & 1 consumed
-      if (j + 2 < n_chunks) stage_issue(j + 2, kc, vc);
+      __syncthreads();  // buffer j % kNB consumed
+      if (j + kNB < n_chunks) stage_issue(j + kNB, kc, vc);
+    }
+    if (tid == 0) {  // every staged row has landed and been read: gate/up, W_d into slots 2-5
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      for (int i = kPersistAChunks; i < kLayerChunks; ++i) issue(q0 + i);
     }
     if (warp < 6 && own_n > 0)
       attend(reinterpret_cast<const unsigned char*>(ownk + static_cast<size_t>(own_lo) * kQS),
              reinterpret_cast<const unsigned char*>(ownv + static_cast<size_t>(own_lo) * kQS), kQS * 2, own_n);
+
+    // --- merge the two key halves of each query tile: warp (qt, kh) keeps value dims
+    // 64 kh .. 64 kh + 63. It hands the other 64 dims of its accumulator and its running
+    // max / sum to its partner through the activation image (idle now; thread-fragment
+    // order, so every lane reads back exactly its partner lane's values).
+    float o_fin[8][4];
+    {
+      float4* xo = reinterpret_cast<float4*>(act);   // [3 qt][2 kh][8][32 lanes]
+      float4* xml = xo + 3 * 2 * 8 * 32;              // [3 qt][2 kh][32 lanes]: m0, m1, l0, l1
+      if (warp < 6) {
+#pragma unroll
+        for (int nb = 0; nb < 8; ++nb) {
+          const float* src = kh == 0 ? o_acc[8 + nb] : o_acc[nb];
+          xo[((qt * 2 + kh) * 8 + nb) * 32 + lane] = make_float4(src[0], src[1], src[2], src[3]);
+        }
+        xml[(qt * 2 + kh) * 32 + lane] = make_float4(m_run[0], m_run[1], l_run[0], l_run[1]);
+      }
+      __syncthreads();
+      if (warp < 6) {
+        const int pk = 1 - kh;
+        const float4 pml = xml[(qt * 2 + pk) * 32 + lane];
+        const float pm[2] = {pml.x, pml.y};
+        const float pl[2] = {pml.z, pml.w};
+        float sa[2], sb[2];
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const float m = fmaxf(m_run[r], pm[r]);
+          sa[r] = m == -CUDART_INF_F ? 0.f : exp2f(m_run[r] - m);
+          sb[r] = m == -CUDART_INF_F ? 0.f : exp2f(pm[r] - m);
+          l_run[r] = l_run[r] * sa[r] + pl[r] * sb[r];
+          m_run[r] = m;
+        }
+#pragma unroll
+        for (int nb = 0; nb < 8; ++nb) {
+          const float4 po = xo[((qt * 2 + pk) * 8 + nb) * 32 + lane];
+          const float* mine = kh == 0 ? o_acc[nb] : o_acc[8 + nb];
+          o_fin[nb][0] = mine[0] * sa[0] + po.x * sb[0];
+          o_fin[nb][1] = mine[1] * sa[0] + po.y * sb[0];
+          o_fin[nb][2] = mine[2] * sa[1] + po.z * sb[1];
+          o_fin[nb][3] = mine[3] * sa[1] + po.w * sb[1];
+        }
+      }
+    }
 
     // --- merge the 4 splits: every row's normalised fp32 partial and log-sum-exp go
     // straight from the registers to the rank that owns the row
@@ -718,12 +789,12 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       float* d0 = recv + (rank * kRowsPerRank + qr0 - own0 * kRowsPerRank) * kD;
       float* d1 = recv + (rank * kRowsPerRank + qr1 - own1 * kRowsPerRank) * kD;
 #pragma unroll
-      for (int n = 0; n < 8; ++n) {
-        const int c = dh * 64 + n * 8 + 2 * (lane & 3);
-        st_cluster_v2f(cluster_addr(d0 + c, own0), o_acc[n][0] * inv0, o_acc[n][1] * inv0);
-        st_cluster_v2f(cluster_addr(d1 + c, own1), o_acc[n][2] * inv1, o_acc[n][3] * inv1);
+      for (int nb = 0; nb < 8; ++nb) {
+        const int c = kh * 64 + nb * 8 + 2 * (lane & 3);
+        st_cluster_v2f(cluster_addr(d0 + c, own0), o_fin[nb][0] * inv0, o_fin[nb][1] * inv0);
+        st_cluster_v2f(cluster_addr(d1 + c, own1), o_fin[nb][2] * inv1, o_fin[nb][3] * inv1);
       }
-      if (dh == 0 && (lane & 3) == 0) {
+      if (kh == 0 && (lane & 3) == 0) {
         st_cluster_f32(cluster_addr(recv_lse + rank * kRowsPerRank + qr0 - own0 * kRowsPerRank, own0),
                        l_run[0] > 0.f ? m_run[0] + log2f(l_run[0]) : -CUDART_INF_F);
         st_cluster_f32(cluster_addr(recv_lse + rank * kRowsPerRank + qr1 - own1 * kRowsPerRank, own1),
