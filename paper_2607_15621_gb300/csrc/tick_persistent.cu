@@ -284,9 +284,6 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   const uint32_t act_a = smem_addr(act);
 
   const long long Lc = o_hi - o_lo;
-  const long long n_keys = Lc + T;
-  const long long kbeg = n_keys * rank / kCl;
-  const long long kend = n_keys * (rank + 1) / kCl;
 
   float* X0 = p.X;
   const size_t xs = static_cast<size_t>(kTokTile) * d;  // one residual buffer
@@ -468,11 +465,20 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   static_assert(sizeof(CT) == 4 || kStageKeys % (2 * kKeyTile) == 0, "an even number of key tiles per bf16 chunk");
   static_assert(3 * 2 * 8 * 32 * 16 + 3 * 2 * 32 * 16 <= 8 * kActAtom, "key-half merge scratch exceeds the activation image");
   unsigned char* const stage_base = ring + 2 * kSlotBytes;  // the activation image follows the ring
-  const long long c_hi = min(kend, Lc);
-  const int n_cache = c_hi > kbeg ? static_cast<int>(c_hi - kbeg) : 0;  // cache keys of this CTA
+  // Keys of this CTA: the cache in whole staging chunks, split near-evenly over the
+  // cluster (later ranks take the extra chunks; only the last chunk can be short), and
+  // all T own keys on the rank with the fewest cache keys (the last such rank), so that
+  // no rank pays a chunk iteration for a few leftover keys.
+  const long long n_cchunks = (Lc + kStageKeys - 1) / kStageKeys;
+  auto cache_lo = [&](int r) { return min(Lc, n_cchunks * r / kCl * kStageKeys); };
+  int own_rank = 0;
+  for (int r = 1; r < kCl; ++r)
+    if (cache_lo(r + 1) - cache_lo(r) <= cache_lo(own_rank + 1) - cache_lo(own_rank)) own_rank = r;
+  const long long kbeg = cache_lo(rank);                                // first cache key of this CTA
+  const int n_cache = static_cast<int>(cache_lo(rank + 1) - kbeg);      // cache keys of this CTA
   const int n_chunks = (n_cache + kStageKeys - 1) / kStageKeys;
-  const int own_lo = static_cast<int>(max(kbeg, Lc) - Lc);              // own keys of this CTA
-  const int own_n = static_cast<int>(kend - Lc) - own_lo;
+  const int own_lo = 0;                                                 // own keys of this CTA
+  const int own_n = rank == own_rank ? T : 0;
   const size_t tok_bytes = static_cast<size_t>(p.H) * kD * sizeof(CT);  // one token row of all heads
   const size_t head_off = (static_cast<size_t>(o_lo + kbeg) * p.H + head) * kD * sizeof(CT);
   // all threads: 16-byte cp.async copies of chunk j into buffer j % kNB (one commit group)
@@ -502,7 +508,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       cp_async_wait<1>();
     else
       cp_async_wait<0>();
-    __syncthreads();
+    // bf16: a thread converts exactly the units it copied (same unit -> thread map), so
+    // its own wait suffices; fp32 units are regrouped and need every thread's copies
+    if (sizeof(CT) != 2) __syncthreads();
     const int n = min(kStageKeys, n_cache - j * kStageKeys);
     unsigned char* kb = stage_base + (j % kNB) * kBufBytes;
     if (sizeof(CT) == 2) {
@@ -618,7 +626,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     push_rows(ownv + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
     cluster.sync();  // q, own k, own v complete in every CTA
 
-    // --- Eq. 1 over keys [kbeg, kend) of [cache ; own] in 32-key tiles. Warp w < 6
+    // --- Eq. 1 over this CTA's cache keys, then its own keys, in 32-key tiles. Warp w < 6
     // takes query rows 16 (w % 3) .. +15 and every other key tile (tiles kh, kh + 2, ...
     // of a chunk, kh = w / 3) over all 128 value dims; the two key halves of a query
     // tile are merged in shared memory afterwards (log-sum-exp weights).

@@ -60,6 +60,19 @@ def test_tick_bf16_history_sweep(length):
     _parity(fc.Case(synth.EXPERT, [length], "bf16"))
 
 
+@pytest.mark.parametrize("length", [0, 17, 100, 300])
+def test_tick_b1_persistent_ragged_lengths(length):
+    """One vehicle runs as the single-launch persistent tick; cache lengths that leave a
+    short last staging chunk, fewer cache keys than CTAs of a head, or no cache at all."""
+    case = fc.Case(SMALL, [length], "bf16", seed=7 + length)
+    ex = case.expert()
+    try:
+        assert ex.launches(1) == 1
+    finally:
+        ex.close()
+    _parity(case)
+
+
 def test_tick_bf16_b16_ragged():
     """B=16 vehicles with L_b ~ U[96, 480] sharing the expert weights."""
     _parity(fc.Case(synth.EXPERT, synth.cache_lengths("bf16_b16_ragged"), "bf16"))
