@@ -7,7 +7,7 @@ transposed operand -- fails at least one of them.
 
 Sources used: torch library routines in float64 (scaled_dot_product_attention,
 rms_norm, silu, linear, logsumexp), closed forms of the softmax and of RMSNorm,
-and the invariants the method fixes (Sec. 3.1, Eq. 1: one softmax over the
+the hand-derived cases in tests/golden/, and the invariants the method fixes (Sec. 3.1, Eq. 1: one softmax over the
 concatenated keys; backbone cache read-only; vehicles independent).
 """
 from __future__ import annotations
@@ -23,6 +23,7 @@ import torch.nn.functional as F
 
 import oracle
 from oracle import fsx_oracle
+from test_golden import golden_eq1_three_keys, golden_tick_swiglu_closed_form, golden_tick_uniform_attention
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 TINY = dict(n_layers=2, d_model=16, n_heads=2, head_dim=8, d_ff=24,
@@ -331,7 +332,8 @@ PINS = [pin_rms_norm_library, pin_rms_norm_closed_form, pin_silu_library,
         pin_attention_invariants, pin_tick_library_composition, pin_tick_zero_branches,
         pin_tick_zero_gains, pin_tick_uniform_queries, pin_tick_closed_gate,
         pin_tick_vehicle_independence_and_readonly, pin_tick_layer_matching,
-        pin_tick_first_layer_attention]
+        pin_tick_first_layer_attention, golden_eq1_three_keys, golden_tick_uniform_attention,
+        golden_tick_swiglu_closed_form]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=lambda f: f.__name__)
