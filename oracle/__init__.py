@@ -1,4 +1,8 @@
-"""fp64 CPU oracle of the action-expert tick (test infrastructure only).
+"""fp64 CPU oracles (test infrastructure only).
+
+fsx_oracle     the action-expert tick (Sec. 3.1, Eq. 1);
+append_oracle  the backbone's incremental four-token cache append and the
+               monolithic forward it must match (Sec. 1, Sec. 3.3).
 
 Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline / reference
 legs may import this package; the product path never does.
