@@ -206,6 +206,93 @@ fsx_status fsx_attention_noalloc(const void* d_q, long long q_stride,
                                  const int64_t* d_offsets, int B, int n_heads, int head_dim,
                                  int n_splits, void* d_out, float* d_lse, void* stream);
 
+/* ================================================================== cache append
+ * The slow system's incremental forward (Sec. 1, Sec. 3.3): every K = 4 ticks
+ * the current frame's n_new (4) tokens go through the frozen backbone -- a
+ * causal, LLaMA-style decoder -- and every layer appends their keys (after the
+ * rotary embedding) and values to its KV cache, the cache fsx_tick reads. The
+ * cost does not depend on the history length, and rotary phases make the
+ * append exact against a monolithic forward over the whole history.
+ * Per layer, for the new token rows x of one vehicle:
+ *   N = RMSNorm(x; g1, eps 1e-6);  q, k, v = N W_q^T, N W_k^T, N W_v^T;
+ *   q, k rotated at their positions (dims j and j + head_dim/2 of a head turn
+ *   by pos * rope_base^(-2j/head_dim); cached token i of a vehicle sits at
+ *   position i, so the new tokens take positions L_b .. L_b + n_new - 1);
+ *   causal attention over [the vehicle's cached rows ; the new rows];
+ *   x += o W_o^T;  N = RMSNorm(x; g2);  x += (silu(N W_g^T) * (N W_u^T)) W_d^T.
+ * Precision: weights fp16 (RNE from the fp32 host copy), GEMM operands fp16
+ * with fp32 accumulation, fp32 residual stream, RMSNorm, rotation and softmax;
+ * the cache rows are bf16 and the new rows are rounded to bf16 when written. */
+typedef struct fsx_append_s* fsx_append_handle;
+
+typedef struct {
+  int n_layers;              /* backbone layers (32)                                  */
+  int d_model;               /* backbone width (4096), a multiple of 128              */
+  int n_heads;               /* attention heads (32)                                  */
+  int head_dim;              /* head width, must be 128                               */
+  int d_ff;                  /* SwiGLU hidden width (11008), a multiple of 64         */
+  int n_new;                 /* tokens appended per vehicle and call, 1..8 (4)        */
+  int max_batch;             /* largest B of any later call; n_new * max_batch <= 256 */
+  long long max_cache_rows;  /* rows of every K/V cache buffer passed to fsx_append   */
+  float rope_base;           /* rotary base (10000), > 1                              */
+} fsx_append_config;
+
+/* Host fp32 backbone weights, copied (and converted) by fsx_append_create;
+ * every matrix is row-major [out_features, in_features], stacked over layers. */
+typedef struct {
+  const float* attn_norm;  /* [n_layers, d]                     RMSNorm gain, attention */
+  const float* wq;         /* [n_layers, n_heads*head_dim, d]   W_q                     */
+  const float* wk;         /* [n_layers, n_heads*head_dim, d]   W_k                     */
+  const float* wv;         /* [n_layers, n_heads*head_dim, d]   W_v                     */
+  const float* wo;         /* [n_layers, d, n_heads*head_dim]   W_o                     */
+  const float* mlp_norm;   /* [n_layers, d]                     RMSNorm gain, SwiGLU    */
+  const float* w_gate;     /* [n_layers, d_ff, d]               SwiGLU gate             */
+  const float* w_up;       /* [n_layers, d_ff, d]               SwiGLU up               */
+  const float* w_down;     /* [n_layers, d, d_ff]               SwiGLU down             */
+} fsx_append_weights;
+
+/* Create an append handle on `device`: validates cfg (host), uploads fp16
+ * weights in the tensor-core tile order, allocates workspace for
+ * cfg->max_batch vehicles. Blocking. Errors: INVALID_ARG (null pointers,
+ * non-positive fields), UNSUPPORTED (shape outside the list above), OOM, CUDA. */
+fsx_status fsx_append_create(const fsx_append_config* cfg, const fsx_append_weights* w, int device,
+                             fsx_append_handle* out);
+
+/* Append n_new tokens for each of B vehicles.
+ *   k_cache, v_cache : HOST arrays of n_layers DEVICE pointers, none NULL; layer
+ *                      l points to bf16 [max_cache_rows, n_heads, head_dim]
+ *                      rows, token-major. Read, and written only at the rows
+ *                      named by d_dst_rows.
+ *   d_offsets        : DEVICE int64 [B+1], non-decreasing, offsets[0] >= 0,
+ *                      offsets[B] <= max_cache_rows: vehicle b's cached tokens
+ *                      0 .. L_b-1 are rows offsets[b] .. offsets[b+1]-1 (L_b may be 0).
+ *   d_dst_rows       : DEVICE int64 [B]: vehicle b's new rows are written at rows
+ *                      dst[b] .. dst[b] + n_new - 1 of every layer. These ranges
+ *                      must lie in [0, max_cache_rows), must not overlap each
+ *                      other, and must not overlap [offsets[0], offsets[B]).
+ *   B                : 1 .. max_batch.
+ *   d_x_new          : DEVICE bf16 [B, n_new, d] embeddings of the new tokens.
+ *   d_hidden         : DEVICE fp32 [B, n_new, d] output: the residual stream
+ *                      after the last layer (no final norm).
+ * Enqueued on `stream` (kernel by kernel, no host synchronisation). The
+ * device-side checks of offsets and destination rows set a sticky status read
+ * by fsx_append_get_status; such a call writes no cache row and leaves d_hidden
+ * undefined. A handle must not run two appends concurrently, and an append must
+ * not run concurrently with a tick that reads the rows it writes. */
+fsx_status fsx_append(fsx_append_handle h, void* const* k_cache, void* const* v_cache,
+                      const int64_t* d_offsets, const int64_t* d_dst_rows, int B,
+                      const void* d_x_new, float* d_hidden, void* stream);
+
+/* Synchronises `stream`, then returns and clears the handle's device status
+ * word (FSX_OK or FSX_ERR_DEVICE_ARG). */
+fsx_status fsx_append_get_status(fsx_append_handle h, void* stream);
+
+/* Bytes of the handle's fp16 weight arena (algorithmic weight bytes per call). */
+long long fsx_append_weight_bytes(fsx_append_handle h);
+
+/* Releases the handle's device memory (synchronises its device). */
+void fsx_append_destroy(fsx_append_handle h);
+
 #ifdef __cplusplus
 }
 #endif

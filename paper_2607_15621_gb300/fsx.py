@@ -52,6 +52,19 @@ class Weights(ctypes.Structure):
     _fields_ = [(name, ctypes.POINTER(ctypes.c_float)) for name in _WEIGHT_FIELDS]
 
 
+class AppendConfig(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int), ("d_model", ctypes.c_int), ("n_heads", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("d_ff", ctypes.c_int), ("n_new", ctypes.c_int),
+                ("max_batch", ctypes.c_int), ("max_cache_rows", ctypes.c_longlong), ("rope_base", ctypes.c_float)]
+
+
+_APPEND_WEIGHT_FIELDS = ["attn_norm", "wq", "wk", "wv", "wo", "mlp_norm", "w_gate", "w_up", "w_down"]
+
+
+class AppendWeights(ctypes.Structure):
+    _fields_ = [(name, ctypes.POINTER(ctypes.c_float)) for name in _APPEND_WEIGHT_FIELDS]
+
+
 def _load():
     if not os.path.exists(LIB_PATH):
         raise RuntimeError(f"{LIB_PATH} is missing: build it with paper_2607_15621_gb300.build.build()")
@@ -76,6 +89,12 @@ def _load():
                                 vp, i32, i32, i32, i32, vp, vp, vp, ctypes.c_size_t, vp]),
         "fsx_attention_noalloc": (i32, [vp, ctypes.c_longlong, vp, vp, ctypes.c_longlong, i32, i32, vp, vp,
                                         i32, vp, i32, i32, i32, i32, vp, vp, vp]),
+        "fsx_append_create": (i32, [ctypes.POINTER(AppendConfig), ctypes.POINTER(AppendWeights), i32,
+                                    ctypes.POINTER(vp)]),
+        "fsx_append": (i32, [vp, vpp, vpp, vp, vp, i32, vp, vp, vp]),
+        "fsx_append_get_status": (i32, [vp, vp]),
+        "fsx_append_weight_bytes": (ctypes.c_longlong, [vp]),
+        "fsx_append_destroy": (None, [vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -97,7 +116,9 @@ def lib():
 def declared_symbols() -> list[str]:
     return ["fsx_create", "fsx_tick", "fsx_tick_host", "fsx_tick_debug", "fsx_get_status", "fsx_last_error",
             "fsx_destroy", "fsx_weight_bytes", "fsx_tick_launches", "fsx_set_kernel_timing",
-            "fsx_kernel_time", "fsx_attention_workspace_bytes", "fsx_attention", "fsx_attention_noalloc"]
+            "fsx_kernel_time", "fsx_attention_workspace_bytes", "fsx_attention", "fsx_attention_noalloc",
+            "fsx_append_create", "fsx_append", "fsx_append_get_status", "fsx_append_weight_bytes",
+            "fsx_append_destroy"]
 
 
 def last_error() -> str:
@@ -235,3 +256,42 @@ def attention_noalloc(q, q_stride, k_own, v_own, own_stride, n_q, n_own, k_cache
                                       _ptr(k_cache), _ptr(v_cache), code, _ptr(offsets), B, n_heads, 128,
                                       n_splits, _ptr(out), _ptr(lse), _stream(stream)))
     return out
+
+
+class Append:
+    """Owns one fsx_append handle: the backbone's incremental cache append
+    (weights uploaded at construction). Argument marshalling only."""
+
+    def __init__(self, dims, weights: dict, max_batch: int, max_cache_rows: int, device: int = 0):
+        self.dims = dims
+        self.cfg = AppendConfig(dims.n_layers, dims.d_model, dims.n_heads, dims.head_dim, dims.d_ff, dims.n_new,
+                                max_batch, max_cache_rows, float(dims.rope_base))
+        keep = {k: np.ascontiguousarray(weights[k], dtype=np.float32) for k in _APPEND_WEIGHT_FIELDS}
+        wst = AppendWeights(*[keep[k].ctypes.data_as(ctypes.POINTER(ctypes.c_float)) for k in _APPEND_WEIGHT_FIELDS])
+        h = ctypes.c_void_p()
+        check(lib().fsx_append_create(ctypes.byref(self.cfg), ctypes.byref(wst), device, ctypes.byref(h)))
+        self.h = h
+        del keep
+
+    def close(self):
+        if getattr(self, "h", None) and self.h.value:
+            lib().fsx_append_destroy(self.h)
+            self.h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def append(self, k_layers, v_layers, offsets, dst_rows, x_new, hidden, stream=None):
+        B = int(x_new.shape[0])
+        check(lib().fsx_append(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(offsets), _ptr(dst_rows), B,
+                               _ptr(x_new), _ptr(hidden), _stream(stream)))
+        return hidden
+
+    def status(self, stream=None) -> int:
+        return lib().fsx_append_get_status(self.h, _stream(stream))
+
+    def weight_bytes(self) -> int:
+        return int(lib().fsx_append_weight_bytes(self.h))

@@ -52,6 +52,26 @@ class Dims:
 
 EXPERT = Dims()
 
+
+@dataclass(frozen=True)
+class BackboneDims:
+    """Shape of the frozen backbone whose cache the slow system appends to
+    (a LLaMA-7B-shaped causal decoder) and of one append call."""
+    n_layers: int = 32
+    d_model: int = 4096
+    n_heads: int = 32
+    head_dim: int = 128
+    d_ff: int = 11008
+    n_new: int = 4
+    rope_base: float = 10000.0
+
+    @property
+    def hd(self) -> int:
+        return self.n_heads * self.head_dim
+
+
+BACKBONE = BackboneDims()
+
 # Workloads: name -> (batch, length spec, dtype). Length spec is either a fixed
 # per-vehicle cache length or a (lo, hi) inclusive uniform range.
 WORKLOADS = {
@@ -69,6 +89,8 @@ _STREAM_WEIGHTS = 0x5EED0001
 _STREAM_CACHE = 0x5EED0002
 _STREAM_FRAMES = 0x5EED0003
 _STREAM_LENGTHS = 0x5EED0004
+_STREAM_BACKBONE = 0x5EED0005
+_STREAM_APPEND_TOKENS = 0x5EED0006
 
 
 def _gen(seed: int, stream: int, device="cpu") -> torch.Generator:
@@ -160,3 +182,34 @@ def make_frames(dims: Dims, batch: int, seed: int = 0, dtype: str = "bf16", devi
 def as_f64(t: torch.Tensor) -> np.ndarray:
     """Exact fp64 copy of a (possibly bf16 / device) tensor for the oracle."""
     return t.detach().to("cpu", torch.float64).numpy()
+
+
+def make_backbone_weights(dims: BackboneDims = BACKBONE, seed: int = 0, dtype: str = "bf16") -> dict:
+    """Backbone weights as C-contiguous float32 numpy arrays, stacked over layers,
+    [out_features, in_features]: W ~ N(0, 1/fan_in), norm gains ~ 1 + 0.1 N(0, 1)."""
+    g = _gen(seed, _STREAM_BACKBONE)
+    nl, d, hd, f = dims.n_layers, dims.d_model, dims.hd, dims.d_ff
+
+    def normal(shape, std):
+        return torch.randn(*shape, generator=g, dtype=torch.float32) * std
+
+    w = {
+        "attn_norm": 1.0 + normal((nl, d), 0.1),
+        "wq": normal((nl, hd, d), 1.0 / math.sqrt(d)),
+        "wk": normal((nl, hd, d), 1.0 / math.sqrt(d)),
+        "wv": normal((nl, hd, d), 1.0 / math.sqrt(d)),
+        "wo": normal((nl, d, hd), 1.0 / math.sqrt(hd)),
+        "mlp_norm": 1.0 + normal((nl, d), 0.1),
+        "w_gate": normal((nl, f, d), 1.0 / math.sqrt(d)),
+        "w_up": normal((nl, f, d), 1.0 / math.sqrt(d)),
+        "w_down": normal((nl, d, f), 1.0 / math.sqrt(f)),
+    }
+    return {k: np.ascontiguousarray(_round(v, dtype).numpy()) for k, v in w.items()}
+
+
+def make_append_tokens(dims: BackboneDims, batch: int, seed: int = 0, device="cpu"):
+    """Embeddings of the tokens one append call adds, bf16 [B, n_new, d] ~ N(0, 1)."""
+    dev = torch.device(device)
+    g = _gen(seed, _STREAM_APPEND_TOKENS, device=dev.type if dev.type == "cpu" else dev)
+    x = torch.randn(batch, dims.n_new, dims.d_model, generator=g, device=dev)
+    return x.to(torch.bfloat16).contiguous()

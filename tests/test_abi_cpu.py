@@ -139,3 +139,68 @@ def test_attention_host_validation(lib):
     assert call(qs=4095) == fsx.FSX_ERR_INVALID_ARG
     assert call(dt=3) == fsx.FSX_ERR_INVALID_ARG
     assert "workspace" in fsx.last_error() or fsx.last_error()
+
+
+# ---------------------------------------------------------------- cache append
+def _append_cfg(**over):
+    d = synth.BackboneDims(n_layers=1, d_model=128, n_heads=1, d_ff=64)
+    cfg = fsx.AppendConfig(d.n_layers, d.d_model, d.n_heads, d.head_dim, d.d_ff, d.n_new, 4, 1000,
+                           float(d.rope_base))
+    for k, v in over.items():
+        setattr(cfg, k, v)
+    return cfg
+
+
+def _append_create(lib, cfg, weights=True):
+    keep = None
+    if weights:
+        w = synth.make_backbone_weights(synth.BackboneDims(n_layers=1, d_model=128, n_heads=1, d_ff=64), 0)
+        keep = {k: np.ascontiguousarray(w[k], dtype=np.float32) for k in fsx._APPEND_WEIGHT_FIELDS}
+        wst = fsx.AppendWeights(*[keep[k].ctypes.data_as(ctypes.POINTER(ctypes.c_float))
+                                  for k in fsx._APPEND_WEIGHT_FIELDS])
+        wp = ctypes.byref(wst)
+    else:
+        wp = None
+    h = ctypes.c_void_p()
+    st = lib.fsx_append_create(ctypes.byref(cfg) if cfg is not None else None, wp, 0, ctypes.byref(h))
+    return st, h
+
+
+def test_append_create_rejects_null_arguments(lib):
+    st, h = _append_create(lib, None)
+    assert st == fsx.FSX_ERR_INVALID_ARG and not h.value
+    assert "config" in fsx.last_error()
+    st, h = _append_create(lib, _append_cfg(), weights=False)
+    assert st == fsx.FSX_ERR_INVALID_ARG and not h.value
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("head_dim", 64, fsx.FSX_ERR_UNSUPPORTED),
+    ("d_model", 200, fsx.FSX_ERR_UNSUPPORTED),
+    ("d_ff", 100, fsx.FSX_ERR_UNSUPPORTED),
+    ("n_new", 9, fsx.FSX_ERR_UNSUPPORTED),
+    ("max_batch", 65, fsx.FSX_ERR_UNSUPPORTED),
+    ("n_layers", 0, fsx.FSX_ERR_INVALID_ARG),
+    ("max_cache_rows", -1, fsx.FSX_ERR_INVALID_ARG),
+    ("rope_base", 1.0, fsx.FSX_ERR_INVALID_ARG),
+])
+def test_append_create_rejects_bad_shapes(lib, field, value, code):
+    st, h = _append_create(lib, _append_cfg(**{field: value}))
+    assert st == code, fsx.last_error()
+    assert not h.value
+    assert fsx.last_error()
+
+
+def test_append_create_without_gpu_reports_cuda_error(lib):
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    st, h = _append_create(lib, _append_cfg())
+    assert st == fsx.FSX_ERR_CUDA and not h.value
+
+
+def test_append_rejects_null_handle(lib):
+    arr = (ctypes.c_void_p * 1)()
+    assert lib.fsx_append(None, arr, arr, 1, 1, 1, 1, 1, None) == fsx.FSX_ERR_INVALID_ARG
+    assert lib.fsx_append_get_status(None, None) == fsx.FSX_ERR_INVALID_ARG
+    assert lib.fsx_append_weight_bytes(None) == 0
+    lib.fsx_append_destroy(None)  # no-op
