@@ -4,6 +4,10 @@ head) on synthetic seeded inputs, printed as one JSON line.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl fsx|reference]
 
+The workload `append_b1_l224` instead times the backbone's incremental cache
+append (one call = n_new = 4 tokens through the 32-layer, 4096-wide backbone
+for one vehicle with 224 cached tokens); value = vehicle-appends/s.
+
 Default workload: bf16_b1_l224 (B=1 vehicle, 224 cached backbone tokens per
 layer = 64 instruction + 40 frames x 4, bf16 weights/cache/frames, 32 layers).
 value = vehicle-ticks/s over all ranks (weak scaling: every rank runs its own
@@ -185,6 +189,171 @@ def cpu_baseline(name, seconds):
             "sample": f"{n} full 32-layer fp64 ticks of vehicle 0 of {name} (L={int(lengths[0])}) in {el:.1f} s"}
 
 
+APPEND_METRIC = "vehicle-appends/s (1e6 / us-per-append x B) of the backbone's incremental cache append"
+APPEND_UNIT = "vehicle-appends/s"
+
+
+def append_inputs(args, device):
+    """Backbone dims, weights, per-layer caches (cached rows then room for the new
+    rows), offsets, destination rows and new-token embeddings of an append workload."""
+    import torch
+    from paper_2607_15621_gb300 import synth
+    spec = synth.APPEND_WORKLOADS[args.workload]
+    dims = synth.BACKBONE if args.layers is None else dataclasses.replace(synth.BACKBONE, n_layers=args.layers)
+    B, L, n = spec["batch"], spec["length"], dims.n_new
+    w = synth.make_backbone_weights(dims, 0, "bf16")
+    cache_dims = synth.Dims(n_layers=dims.n_layers, n_heads=dims.n_heads, head_dim=dims.head_dim)
+    k, v, off = synth.make_cache(cache_dims, [L] * B, 0, "bf16", device=device)
+    rows = B * (L + n)
+    kc, vc = [], []
+    for kl, vl in zip(k, v):
+        kt = torch.zeros(rows, dims.n_heads, dims.head_dim, dtype=torch.bfloat16, device=device)
+        vt = torch.zeros_like(kt)
+        kt[:B * L] = kl
+        vt[:B * L] = vl
+        kc.append(kt)
+        vc.append(vt)
+    dst = np.array([B * L + n * b for b in range(B)], dtype=np.int64)
+    x = synth.make_append_tokens(dims, B, 0, device=device)
+    return dims, w, kc, vc, off, dst, x, B, L
+
+
+def append_cpu_baseline(args, dims, w, kc, vc, off, x, seconds):
+    """The fp64 append oracle as it stands, on the host cores: vehicle 0's append."""
+    from oracle import append_oracle
+    lo, hi = int(off[0]), int(off[1])
+    kn = [t[lo:hi].float().cpu().numpy() for t in kc]
+    vn = [t[lo:hi].float().cpu().numpy() for t in vc]
+    xn = x[:1].float().cpu().numpy()
+    n, t0 = 0, time.perf_counter()
+    while True:
+        append_oracle.backbone_append(w, kn, vn, np.array([0, hi - lo]), xn, dims.n_heads, dims.head_dim)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or n >= 1000:
+            break
+    return {"value": n / el, "unit": APPEND_UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{n} full {dims.n_layers}-layer fp64 appends of vehicle 0 of {args.workload} "
+                      f"(L={hi - lo}) in {el:.1f} s"}
+
+
+def run_append_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    dims, w, kc, vc, off, dst, x, B, L = append_inputs(args, "cpu")
+    cb = append_cpu_baseline(args, dims, w, kc, vc, off, x, max(1.0, min(args.cpu_seconds, 60.0)))
+    line = {"impl": "reference", "metric": APPEND_METRIC, "value": cb["value"], "unit": APPEND_UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / cb["value"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded)",
+            "config": {"workload": args.workload, "B": B, "cache_len": L, "layers": dims.n_layers,
+                       "d_model": dims.d_model, "new_tokens": dims.n_new, "parallelism": f"replicas x{world}",
+                       "sample": "vehicle 0 per step; vehicles are independent"},
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": APPEND_UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def run_append(args):
+    """The cache append on the GPU: CUDA events around K calls, inputs resident in HBM."""
+    import torch
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2607_15621_gb300 import fsx
+    dims, w, kc, vc, off, dst, x, B, L = append_inputs(args, dev)
+    rows = kc[0].shape[0]
+    offsets = torch.as_tensor(off, device=dev)
+    dst_t = torch.as_tensor(dst, device=dev)
+    hidden = torch.empty(B, dims.n_new, dims.d_model, device=dev)
+    ap = fsx.Append(dims, w, B, rows, device=local)
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    # every call writes the same destination rows, so each timed call is a full append
+    for _ in range(max(args.warmup, 3)):
+        ap.append(kc, vc, offsets, dst_t, x, hidden, stream)
+    torch.cuda.synchronize()
+    if ap.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during warm-up")
+    clock_path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")
+    os.makedirs(os.path.dirname(clock_path), exist_ok=True)
+    proc, fh = start_clock_sampler(clock_path, local)
+    time.sleep(0.5)
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        ap.append(kc, vc, offsets, dst_t, x, hidden, stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    ms = max_over_ranks(e0.elapsed_time(e1), dev)
+    clocks = stop_clock_sampler(proc, fh, clock_path)
+    if ap.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during the timed region")
+    ms_per_step = ms / args.steps
+
+    # end to end: new-token embeddings in from pinned host memory, hidden states back
+    x_h = x.cpu().pin_memory()
+    hid_h = torch.empty(B, dims.n_new, dims.d_model).pin_memory()
+    e2e_steps = max(1, args.steps // 2)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        x.copy_(x_h, non_blocking=True)
+        ap.append(kc, vc, offsets, dst_t, x, hidden, stream)
+        hid_h.copy_(hidden, non_blocking=True)
+        stream.synchronize()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
+
+    hbm, tensor_tfs, peak_kind = peaks()
+    hd = dims.hd
+    per_layer_w = 3 * hd * dims.d_model + dims.d_model * hd + 3 * dims.d_ff * dims.d_model
+    cache_bytes = B * (L + dims.n_new) * dims.n_layers * 2 * hd * 2   # cached rows read + new rows written
+    call_bytes = ap.weight_bytes() + cache_bytes
+    flops = (2 * B * dims.n_new * per_layer_w + 4 * B * dims.n_new * hd * (L + dims.n_new)) * dims.n_layers
+    achieved = call_bytes / (ms_per_step / 1e3) / 1e9
+    rl_us = max(call_bytes / (hbm * 1e9), flops / (tensor_tfs * 1e12)) * 1e6
+    line = {
+        "metric": APPEND_METRIC, "value": world * B / (ms_per_step / 1e3), "unit": APPEND_UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_per_step,
+        "us_per_append": ms_per_step * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f16 (fp32 accumulate)", "data": "synthetic (seeded N(0,1/fan_in) weights, N(0,1) cache and tokens)",
+        "config": {"workload": args.workload, "B": B, "cache_len": L, "layers": dims.n_layers,
+                   "d_model": dims.d_model, "new_tokens": dims.n_new,
+                   "l2": "inputs larger than L2 (the backbone weights exceed 129 MB)",
+                   "parallelism": f"replicas x{world}"},
+        "gpu_launches": (1 + 7 * dims.n_layers) * args.steps,
+        "roofline": {"bound": "hbm", "kernel": "append (whole call)", "achieved": achieved, "peak": hbm,
+                     "unit": "GB/s", "frac": achieved / hbm, "traffic": None, "peak_source": peak_kind,
+                     "bytes_per_launch": call_bytes, "launch_us": ms_per_step * 1e3,
+                     "flops_per_call": flops, "roofline_us": rl_us},
+        "e2e": {"value": world * B * e2e_steps / e2e_s, "unit": APPEND_UNIT,
+                "h2d_bytes_per_step": int(x_h.numel() * x_h.element_size()),
+                "d2h_bytes_per_step": int(hid_h.numel() * hid_h.element_size())},
+        "clocks": clocks,
+    }
+    ap.close()
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = append_cpu_baseline(args, dims, w, kc, vc, off, x, args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def run_reference(args):
     world, rank, _ = dist_env()
     if rank != 0:
@@ -205,6 +374,10 @@ def run_reference(args):
 
 def main():
     args = parse()
+    from paper_2607_15621_gb300 import synth
+    if args.workload in synth.APPEND_WORKLOADS:
+        (run_append_reference if args.impl == "reference" else run_append)(args)
+        return
     if args.impl == "reference":
         run_reference(args)
         return

@@ -72,6 +72,12 @@ class BackboneDims:
 
 BACKBONE = BackboneDims()
 
+# Cache-append workloads: one call appends n_new tokens for each of `batch`
+# vehicles, each with `length` cached tokens (64 instruction + 40 frames x 4).
+APPEND_WORKLOADS = {
+    "append_b1_l224": dict(batch=1, length=224),
+}
+
 # Workloads: name -> (batch, length spec, dtype). Length spec is either a fixed
 # per-vehicle cache length or a (lo, hi) inclusive uniform range.
 WORKLOADS = {

@@ -65,3 +65,18 @@ def test_reference_arm_under_torchrun_prints_on_rank0_only():
     assert line["impl"] == "reference"
     assert line["n_gpus"] == 2 and line["unit"] == "vehicle-ticks/s" and line["value"] > 0
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_append_reference_arm_prints_one_line():
+    """The cache-append workload's reference arm: the fp64 append oracle on the host cores
+    (one backbone layer here to keep the CPU suite short)."""
+    cmd = [sys.executable, "bench.py", "--impl", "reference", "--workload", "append_b1_l224", "--layers", "1",
+           "--steps", "1", "--warmup", "1", "--cpu-seconds", "1"]
+    res = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600)
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [l for l in res.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, res.stdout
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["unit"] == "vehicle-appends/s" and line["value"] > 0
+    assert line["config"]["workload"] == "append_b1_l224" and line["config"]["layers"] == 1
+    assert line["cpu_baseline"]["kind"] == "oracle"
