@@ -112,39 +112,22 @@ def _layer(params: dict, layer: int, name: str) -> np.ndarray:
     return np.asarray(params[name][layer], dtype=np.float64)
 
 
-def expert_tick(params: dict, k_cache, v_cache, offsets, frames,
-                n_heads: int, head_dim: int, n_waypoints: int = 5,
-                capture_attention: bool = False):
-    """One expert tick for B vehicles (Sec. 3.1, Eq. 1; Sec. 3.3 deployment).
+def expert_layers(params: dict, x: np.ndarray, k_cache, v_cache, offsets, n_heads: int, head_dim: int,
+                  capture_attention: bool = False):
+    """The expert's layer stack (Sec. 3.1, Eq. 1) on assembled tokens x [B, T, d].
 
-    params: dict of arrays (any float dtype; read as fp64), stacked over layers:
-      act_emb [n_action, d], pos_emb [n_action + n_frame, d],
+    params: stacked over layers, matrices [out_features, in_features]:
       attn_norm [NL, d], wq/wk/wv [NL, H*D, d], wo [NL, d, H*D],
-      mlp_norm [NL, d], w_gate/w_up [NL, F, d], w_down [NL, d, F],
-      final_norm [d], head_w [2, d], head_b [2]
-      (every matrix is [out_features, in_features]).
+      mlp_norm [NL, d], w_gate/w_up [NL, F, d], w_down [NL, d, F].
     k_cache, v_cache: sequence of NL arrays [total_tokens, H, D]; vehicle b owns
       rows offsets[b] .. offsets[b+1]-1 of every layer. They are only read.
-    offsets: [B+1] non-decreasing integers.
-    frames: [B, n_frame, d] frame tokens.
-
-    Returns waypoints [B, n_waypoints, 2] (fp64) and, if capture_attention,
-    also A [NL, B*T, H*D]: each layer's Eq. 1 output before W_o, token-major.
-    """
-    act_emb = np.asarray(params["act_emb"], np.float64)
-    pos_emb = np.asarray(params["pos_emb"], np.float64)
-    frames = np.asarray(frames, np.float64)
+    Returns the residual stream after the last layer [B, T, d] and, if
+    capture_attention, A [NL, B*T, H*D]: each layer's Eq. 1 output before W_o."""
+    x = np.array(x, dtype=np.float64)
     offsets = np.asarray(offsets, dtype=np.int64)
-    n_batch = frames.shape[0]
+    n_batch, n_tok, _ = x.shape
     n_layers = len(params["wq"])
-    n_tok = act_emb.shape[0] + frames.shape[1]
     hd = n_heads * head_dim
-
-    # token assembly: learned action tokens, then the frame tokens, plus the
-    # learned positional embedding (expert tokens carry no rotary phase)
-    x = np.concatenate([np.broadcast_to(act_emb, (n_batch,) + act_emb.shape), frames], axis=1)
-    x = x + pos_emb[None, :, :]                                   # [B, T, d]
-
     captured = np.zeros((n_layers, n_batch * n_tok, hd)) if capture_attention else None
     for layer in range(n_layers):
         wq = _layer(params, layer, "wq")
@@ -172,6 +155,33 @@ def expert_tick(params: dict, k_cache, v_cache, offsets, frames,
             x[b] = x[b] + a @ wo.T
             n = rms_norm(x[b], g2)
             x[b] = x[b] + (silu(n @ wg.T) * (n @ wu.T)) @ wd.T
+    return x, captured
+
+
+def expert_tick(params: dict, k_cache, v_cache, offsets, frames,
+                n_heads: int, head_dim: int, n_waypoints: int = 5,
+                capture_attention: bool = False):
+    """One expert tick for B vehicles (Sec. 3.1, Eq. 1; Sec. 3.3 deployment).
+
+    params: dict of arrays (any float dtype; read as fp64): the layer weights of
+      expert_layers plus act_emb [n_action, d], pos_emb [n_action + n_frame, d],
+      final_norm [d], head_w [2, d], head_b [2].
+    k_cache, v_cache, offsets: as in expert_layers.
+    frames: [B, n_frame, d] frame tokens.
+
+    Returns waypoints [B, n_waypoints, 2] (fp64) and, if capture_attention,
+    also A [NL, B*T, H*D]: each layer's Eq. 1 output before W_o, token-major.
+    """
+    act_emb = np.asarray(params["act_emb"], np.float64)
+    pos_emb = np.asarray(params["pos_emb"], np.float64)
+    frames = np.asarray(frames, np.float64)
+    n_batch = frames.shape[0]
+
+    # token assembly: learned action tokens, then the frame tokens, plus the
+    # learned positional embedding (expert tokens carry no rotary phase)
+    x = np.concatenate([np.broadcast_to(act_emb, (n_batch,) + act_emb.shape), frames], axis=1)
+    x = x + pos_emb[None, :, :]                                   # [B, T, d]
+    x, captured = expert_layers(params, x, k_cache, v_cache, offsets, n_heads, head_dim, capture_attention)
 
     head_w = np.asarray(params["head_w"], np.float64)
     head_b = np.asarray(params["head_b"], np.float64)
