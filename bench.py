@@ -124,6 +124,13 @@ def tick_flops(dims, lengths):
     return gemm + attn
 
 
+def clock_dir():
+    """Where the raw nvidia-smi samples of the timed region go (FSX_CLOCKS_DIR, else a
+    temporary directory); the JSON line carries their summary."""
+    import tempfile
+    return os.environ.get("FSX_CLOCKS_DIR") or tempfile.gettempdir()
+
+
 def start_clock_sampler(path, index):
     try:
         fh = open(path, "w")
@@ -284,7 +291,7 @@ def run_append(args):
     torch.cuda.synchronize()
     if ap.status(stream) != fsx.FSX_OK:
         raise RuntimeError("device status set during warm-up")
-    clock_path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")
+    clock_path = os.path.join(clock_dir(), f"clocks_rank{rank}.csv")
     os.makedirs(os.path.dirname(clock_path), exist_ok=True)
     proc, fh = start_clock_sampler(clock_path, local)
     time.sleep(0.5)
@@ -414,7 +421,7 @@ def main():
     if ex.status(stream) != fsx.FSX_OK:
         raise RuntimeError("device status set during warm-up")
 
-    clock_path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")
+    clock_path = os.path.join(clock_dir(), f"clocks_rank{rank}.csv")
     os.makedirs(os.path.dirname(clock_path), exist_ok=True)
     proc, fh = start_clock_sampler(clock_path, local)
     time.sleep(0.5)
