@@ -114,6 +114,19 @@ fsx_status fsx_tick(fsx_handle h, const void* const* k_cache, const void* const*
                     const int64_t* d_offsets, int B, const void* d_frames,
                     float* d_waypoints, void* stream);
 
+/* fsx_tick with an explicit first row per vehicle, for caches whose vehicles do not
+ * lie back to back: vehicle b reads rows d_starts[b] .. d_starts[b] + L_b - 1 with
+ * L_b = offsets[b+1] - offsets[b]. The ranges may leave gaps (room for the slow
+ * system's appends) or overlap (prefixes of one shared cache, as in the
+ * staleness-masked forward over a clip, Sec. 3.2). d_starts: DEVICE int64 [B], each
+ * >= 0 with d_starts[b] + L_b <= max_total_cache_tokens (checked on the device);
+ * d_offsets: DEVICE int64 [B+1], non-decreasing, giving only the lengths here (its
+ * last entry may exceed max_total_cache_tokens). NULL d_starts is fsx_tick.
+ * Everything else as fsx_tick. */
+fsx_status fsx_tick_ranges(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                           const int64_t* d_starts, const int64_t* d_offsets, int B, const void* d_frames,
+                           float* d_waypoints, void* stream);
+
 /* fsx_tick with HOST frames, offsets and waypoints: copies h_offsets [B+1]
  * and h_frames [B, n_frame, d] to handle-owned device buffers, runs the
  * tick, copies the waypoints back to h_waypoints [B, n_waypoints, 2] and
@@ -128,6 +141,11 @@ fsx_status fsx_tick_host(fsx_handle h, const void* const* k_cache, const void* c
 fsx_status fsx_tick_debug(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
                           const int64_t* d_offsets, int B, const void* d_frames,
                           float* d_waypoints, void* d_attn_out, void* stream);
+
+/* fsx_tick_debug with the per-vehicle first rows of fsx_tick_ranges. For tests. */
+fsx_status fsx_tick_ranges_debug(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                                 const int64_t* d_starts, const int64_t* d_offsets, int B, const void* d_frames,
+                                 float* d_waypoints, void* d_attn_out, void* stream);
 
 /* Synchronises `stream`, then returns and clears the device status word
  * (FSX_OK, FSX_ERR_DEVICE_ARG or FSX_ERR_TIMEOUT). */

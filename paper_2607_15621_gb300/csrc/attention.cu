@@ -141,17 +141,19 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
   const CT* kc;
   const CT* vc;
   const int64_t* offs;
+  const int64_t* starts = nullptr;
   if (p.targs != nullptr) {
     kc = static_cast<const CT*>(p.targs->k_cache[p.layer]);
     vc = static_cast<const CT*>(p.targs->v_cache[p.layer]);
     offs = p.targs->offsets;
+    starts = p.targs->starts;
   } else {
     kc = static_cast<const CT*>(p.k_cache);
     vc = static_cast<const CT*>(p.v_cache);
     offs = p.offsets;
   }
-  const long long o_lo = offs[b];
-  const long long o_hi = offs[b + 1];
+  const long long o_lo = starts != nullptr ? starts[b] : offs[b];
+  const long long o_hi = o_lo + (offs[b + 1] - offs[b]);
   if (o_lo < 0 || o_hi < o_lo || o_hi > p.max_total ||
       (o_hi > o_lo && (kc == nullptr || vc == nullptr))) {  // never read outside the caller's cache
     set_status(p.status, kStatusDeviceArg);

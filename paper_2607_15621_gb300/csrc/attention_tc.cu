@@ -203,17 +203,19 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
   const __nv_bfloat16* kc;
   const __nv_bfloat16* vc;
   const int64_t* offs;
+  const int64_t* starts = nullptr;
   if (p.targs != nullptr) {
     kc = static_cast<const __nv_bfloat16*>(p.targs->k_cache[p.layer]);
     vc = static_cast<const __nv_bfloat16*>(p.targs->v_cache[p.layer]);
     offs = p.targs->offsets;
+    starts = p.targs->starts;
   } else {
     kc = static_cast<const __nv_bfloat16*>(p.k_cache);
     vc = static_cast<const __nv_bfloat16*>(p.v_cache);
     offs = p.offsets;
   }
-  const long long o_lo = offs[b];
-  const long long o_hi = offs[b + 1];
+  const long long o_lo = starts != nullptr ? starts[b] : offs[b];
+  const long long o_hi = o_lo + (offs[b + 1] - offs[b]);
   if (o_lo < 0 || o_hi < o_lo || o_hi > p.max_total || (o_hi > o_lo && (kc == nullptr || vc == nullptr))) {
     set_status(p.status, kStatusDeviceArg);  // never read outside the caller's cache
     return;

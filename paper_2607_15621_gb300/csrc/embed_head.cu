@@ -1,7 +1,8 @@
 // Token assembly and waypoint head of the action expert (Sec. 3.1).
 //
 // embed: x_b = [E_act ; F_b] + P_pos into the fp32 residual stream; block 0
-//        also checks the cache offsets (non-decreasing, within capacity) and
+//        also checks the cache ranges (offsets non-decreasing; the rows of every
+//        vehicle, at offsets[b] or at its optional start row, within capacity) and
 //        raises the device status word, which turns the rest of the tick
 //        into no-ops. Block b < B also ranks vehicle b by cache length, so the
 //        attention launches can start the longest caches first (a schedule
@@ -23,9 +24,13 @@ __global__ void embed_kernel(const EmbedArgs a) {
   const int t = row - b * T;
   if (row == 0 && threadIdx.x == 0) {
     const int64_t* off = a.targs->offsets;
+    const int64_t* st = a.targs->starts;
     bool ok = off[0] >= 0;
     for (int i = 0; i < a.B && ok; ++i) ok = off[i + 1] >= off[i];
-    ok = ok && off[a.B] <= a.max_total;
+    if (st == nullptr)
+      ok = ok && off[a.B] <= a.max_total;
+    else  // every vehicle's own row range lies inside the caller's cache
+      for (int i = 0; i < a.B && ok; ++i) ok = st[i] >= 0 && st[i] + (off[i + 1] - off[i]) <= a.max_total;
     if (!ok) set_status(a.status, kStatusDeviceArg);
   }
   __shared__ float s_part[4];

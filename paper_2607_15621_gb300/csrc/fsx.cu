@@ -396,7 +396,8 @@ fsx_status check_tick_args(fsx_handle_s* h, const void* const* k_cache, const vo
 // Upload the per-tick pointers when they changed and order this tick after the
 // previous one if it was issued on another stream.
 fsx_status prepare_tick(fsx_handle_s* h, const void* const* k_cache, const void* const* v_cache,
-                        const int64_t* d_offsets, const void* d_frames, float* d_waypoints, cudaStream_t st) {
+                        const int64_t* d_offsets, const int64_t* d_starts, const void* d_frames, float* d_waypoints,
+                        cudaStream_t st) {
   FSX_CUDA(cudaSetDevice(h->device));
   if (h->has_last && h->last_stream != st) FSX_CUDA(cudaStreamWaitEvent(st, h->last_tick, 0));
   TickArgs a{};
@@ -405,6 +406,7 @@ fsx_status prepare_tick(fsx_handle_s* h, const void* const* k_cache, const void*
     a.v_cache[l] = v_cache[l];
   }
   a.offsets = d_offsets;
+  a.starts = d_starts;
   a.frames = d_frames;
   a.waypoints = d_waypoints;
   if (!h->args_valid || std::memcmp(&a, &h->h_args, sizeof(TickArgs)) != 0) {
@@ -698,13 +700,14 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
   return FSX_OK;
 }
 
-fsx_status fsx_tick(fsx_handle h, const void* const* k_cache, const void* const* v_cache, const int64_t* d_offsets,
-                    int B, const void* d_frames, float* d_waypoints, void* stream) {
+fsx_status fsx_tick_ranges(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                           const int64_t* d_starts, const int64_t* d_offsets, int B, const void* d_frames,
+                           float* d_waypoints, void* stream) {
   fsx_status s = check_tick_args(h, k_cache, v_cache, d_offsets, B, d_frames, d_waypoints);
   if (s != FSX_OK) return s;
   std::lock_guard<std::mutex> lock(h->mu);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  s = prepare_tick(h, k_cache, v_cache, d_offsets, d_frames, d_waypoints, st);
+  s = prepare_tick(h, k_cache, v_cache, d_offsets, d_starts, d_frames, d_waypoints, st);
   if (s != FSX_OK) return s;
   cudaGraphExec_t exec = nullptr;
   s = get_graph(h, B, h->timing, &exec);
@@ -712,6 +715,11 @@ fsx_status fsx_tick(fsx_handle h, const void* const* k_cache, const void* const*
   FSX_CUDA(cudaGraphLaunch(exec, st));
   h->timed_pending = h->timing;
   return finish_tick(h, st);
+}
+
+fsx_status fsx_tick(fsx_handle h, const void* const* k_cache, const void* const* v_cache, const int64_t* d_offsets,
+                    int B, const void* d_frames, float* d_waypoints, void* stream) {
+  return fsx_tick_ranges(h, k_cache, v_cache, nullptr, d_offsets, B, d_frames, d_waypoints, stream);
 }
 
 fsx_status fsx_tick_host(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
@@ -736,19 +744,26 @@ fsx_status fsx_tick_host(fsx_handle h, const void* const* k_cache, const void* c
   return FSX_OK;
 }
 
-fsx_status fsx_tick_debug(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
-                          const int64_t* d_offsets, int B, const void* d_frames, float* d_waypoints,
-                          void* d_attn_out, void* stream) {
+fsx_status fsx_tick_ranges_debug(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                                 const int64_t* d_starts, const int64_t* d_offsets, int B, const void* d_frames,
+                                 float* d_waypoints, void* d_attn_out, void* stream) {
   fsx_status s = check_tick_args(h, k_cache, v_cache, d_offsets, B, d_frames, d_waypoints);
   if (s != FSX_OK) return s;
   if (!d_attn_out) return fail(FSX_ERR_INVALID_ARG, "d_attn_out is NULL");
   std::lock_guard<std::mutex> lock(h->mu);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  s = prepare_tick(h, k_cache, v_cache, d_offsets, d_frames, d_waypoints, st);
+  s = prepare_tick(h, k_cache, v_cache, d_offsets, d_starts, d_frames, d_waypoints, st);
   if (s != FSX_OK) return s;
   s = enqueue_tick(h, B, st, static_cast<__half*>(d_attn_out), false);
   if (s != FSX_OK) return s;
   return finish_tick(h, st);
+}
+
+fsx_status fsx_tick_debug(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                          const int64_t* d_offsets, int B, const void* d_frames, float* d_waypoints,
+                          void* d_attn_out, void* stream) {
+  return fsx_tick_ranges_debug(h, k_cache, v_cache, nullptr, d_offsets, B, d_frames, d_waypoints, d_attn_out,
+                               stream);
 }
 
 fsx_status fsx_get_status(fsx_handle h, void* stream) {

@@ -19,6 +19,10 @@ struct TickArgs {
   const void* k_cache[kMaxLayers];
   const void* v_cache[kMaxLayers];
   const int64_t* offsets;
+  // optional [B]: first cache row of vehicle b; its rows are then starts[b] ..
+  // starts[b] + (offsets[b+1] - offsets[b]) - 1, and the ranges of different
+  // vehicles may overlap or leave gaps (offsets then only give the lengths)
+  const int64_t* starts;
   const void* frames;
   float* waypoints;
 };

@@ -249,8 +249,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
 
   // ---- vehicle 0's cache range, checked once (uniform across the grid)
   const int64_t* offs = p.targs->offsets;
-  const long long o_lo = offs[0];
-  const long long o_hi = offs[1];
+  const long long o_lo = p.targs->starts != nullptr ? p.targs->starts[0] : offs[0];
+  const long long o_hi = o_lo + (offs[1] - offs[0]);
   bool bad = o_lo < 0 || o_hi < o_lo || o_hi > p.max_total;
   if (!bad && o_hi > o_lo)  // a non-empty cache needs every layer's rows
     for (int l = 0; l < p.n_layers; ++l)

@@ -77,6 +77,8 @@ def _load():
         "fsx_tick": (i32, [vp, vpp, vpp, vp, i32, vp, vp, vp]),
         "fsx_tick_host": (i32, [vp, vpp, vpp, vp, i32, vp, vp, vp]),
         "fsx_tick_debug": (i32, [vp, vpp, vpp, vp, i32, vp, vp, vp, vp]),
+        "fsx_tick_ranges": (i32, [vp, vpp, vpp, vp, vp, i32, vp, vp, vp]),
+        "fsx_tick_ranges_debug": (i32, [vp, vpp, vpp, vp, vp, i32, vp, vp, vp, vp]),
         "fsx_get_status": (i32, [vp, vp]),
         "fsx_last_error": (ctypes.c_char_p, []),
         "fsx_destroy": (None, [vp]),
@@ -114,7 +116,8 @@ def lib():
 
 
 def declared_symbols() -> list[str]:
-    return ["fsx_create", "fsx_tick", "fsx_tick_host", "fsx_tick_debug", "fsx_get_status", "fsx_last_error",
+    return ["fsx_create", "fsx_tick", "fsx_tick_host", "fsx_tick_debug", "fsx_tick_ranges", "fsx_tick_ranges_debug",
+            "fsx_get_status", "fsx_last_error",
             "fsx_destroy", "fsx_weight_bytes", "fsx_tick_launches", "fsx_set_kernel_timing",
             "fsx_kernel_time", "fsx_attention_workspace_bytes", "fsx_attention", "fsx_attention_noalloc",
             "fsx_append_create", "fsx_append", "fsx_append_get_status", "fsx_append_weight_bytes",
@@ -194,10 +197,15 @@ class Expert:
         except Exception:
             pass
 
-    def tick(self, k_layers, v_layers, offsets, frames, out, stream=None):
+    def tick(self, k_layers, v_layers, offsets, frames, out, stream=None, starts=None):
+        """One tick; with `starts`, vehicle b reads rows starts[b] .. starts[b] + L_b - 1."""
         B = int(frames.shape[0])
-        check(lib().fsx_tick(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(offsets), B,
-                             _ptr(frames), _ptr(out), _stream(stream)))
+        if starts is None:
+            check(lib().fsx_tick(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(offsets), B,
+                                 _ptr(frames), _ptr(out), _stream(stream)))
+        else:
+            check(lib().fsx_tick_ranges(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(starts),
+                                        _ptr(offsets), B, _ptr(frames), _ptr(out), _stream(stream)))
         return out
 
     def tick_host(self, k_layers, v_layers, offsets_host: np.ndarray, frames_host, out_host: np.ndarray,
@@ -207,10 +215,15 @@ class Expert:
                                   _ptr(frames_host), _ptr(out_host), _stream(stream)))
         return out_host
 
-    def tick_debug(self, k_layers, v_layers, offsets, frames, out, attn_out, stream=None):
+    def tick_debug(self, k_layers, v_layers, offsets, frames, out, attn_out, stream=None, starts=None):
         B = int(frames.shape[0])
-        check(lib().fsx_tick_debug(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(offsets), B,
-                                   _ptr(frames), _ptr(out), _ptr(attn_out), _stream(stream)))
+        if starts is None:
+            check(lib().fsx_tick_debug(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(offsets), B,
+                                       _ptr(frames), _ptr(out), _ptr(attn_out), _stream(stream)))
+        else:
+            check(lib().fsx_tick_ranges_debug(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(starts),
+                                              _ptr(offsets), B, _ptr(frames), _ptr(out), _ptr(attn_out),
+                                              _stream(stream)))
         return out, attn_out
 
     def status(self, stream=None) -> int:
