@@ -4,6 +4,9 @@ head) on synthetic seeded inputs, printed as one JSON line.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl fsx|reference]
 
+The workload `clip_j40_delta1` times the staleness-masked forward over a 40-frame
+clip (Sec. 3.2: every frame block over the cache prefix ending one frame earlier,
+all blocks in one tick over explicit row ranges); value = frame-blocks/s.
 The workload `append_b1_l224` instead times the backbone's incremental cache
 append (one call = n_new = 4 tokens through the 32-layer, 4096-wide backbone
 for one vehicle with 224 cached tokens); value = vehicle-appends/s.
@@ -361,6 +364,160 @@ def run_append(args):
         dist.destroy_process_group()
 
 
+CLIP_METRIC = "frame-blocks/s of the staleness-masked clip forward (all frames of a clip in one tick)"
+CLIP_UNIT = "frame-blocks/s"
+
+
+def clip_inputs(args, device):
+    """Expert dims and weights, the clip's cache (one buffer), the blocks' prefix lengths
+    as offsets, zero start rows and the blocks' frame tokens."""
+    from paper_2607_15621_gb300 import synth
+    c = synth.CLIP_WORKLOADS[args.workload]
+    dims = synth.EXPERT if args.layers is None else dataclasses.replace(synth.EXPERT, n_layers=args.layers)
+    prefix = synth.clip_prefixes(args.workload)
+    rows = c["text"] + c["tokens_per_frame"] * c["frames"]
+    w = synth.make_weights(dims, 0, "bf16")
+    k, v, _ = synth.make_cache(dims, [rows], 0, "bf16", device=device)
+    off = np.concatenate([[0], np.cumsum(prefix)]).astype(np.int64)
+    frames = synth.make_frames(dims, c["frames"], 0, "bf16", device=device)
+    return dims, w, k, v, off, prefix, frames, rows, c
+
+
+def run_clip_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from oracle import staleness_oracle
+    dims, w, k, v, off, prefix, frames, rows, c = clip_inputs(args, "cpu")
+    kn = [t.float().numpy() for t in k]
+    vn = [t.float().numpy() for t in v]
+    fr = frames.double().numpy()
+    n_blocks, t0 = 0, time.perf_counter()
+    seconds = max(1.0, min(args.cpu_seconds, 60.0))
+    # a bounded sample: the clip's blocks from the last (longest prefix) backwards, one
+    # fp64 tick each, until the time is used
+    for j in range(c["frames"] - 1, -1, -1):
+        pj = int(prefix[j])
+        fsx_oracle_tick(w, [t[:pj] for t in kn], [t[:pj] for t in vn], np.array([0, pj]), fr[j:j + 1], dims)
+        n_blocks += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    el = time.perf_counter() - t0
+    cb = {"value": n_blocks / el, "unit": CLIP_UNIT, "cores": os.cpu_count(), "kind": "oracle",
+          "sample": f"{n_blocks} of {c['frames']} frame blocks of {args.workload} (longest prefixes first), "
+                    f"fp64, in {el:.1f} s"}
+    line = {"impl": "reference", "metric": CLIP_METRIC, "value": cb["value"], "unit": CLIP_UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / cb["value"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded)",
+            "config": {"workload": args.workload, "frames": c["frames"], "text": c["text"], "delta": c["delta"],
+                       "layers": dims.n_layers, "parallelism": f"replicas x{world}"},
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": CLIP_UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def fsx_oracle_tick(w, kc, vc, off, frames, dims):
+    from oracle import fsx_oracle
+    return fsx_oracle.expert_tick(w, kc, vc, off, frames, dims.n_heads, dims.head_dim, dims.n_waypoints)
+
+
+def run_clip(args):
+    """All frame blocks of one clip in one ranged tick on the GPU (CUDA events over K ticks)."""
+    import torch
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2607_15621_gb300 import fsx
+    dims, w, k, v, off, prefix, frames, rows, c = clip_inputs(args, dev)
+    J = c["frames"]
+    offsets = torch.as_tensor(off, device=dev)
+    starts = torch.zeros(J, dtype=torch.int64, device=dev)
+    out = torch.empty(J, dims.n_waypoints, 2, device=dev)
+    ex = fsx.Expert(dims, w, J, rows, "bf16", "bf16", device=local)
+    weight_bytes = ex.weight_bytes()
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(max(args.warmup, 3)):
+        ex.tick(k, v, offsets, frames, out, stream, starts=starts)
+    torch.cuda.synchronize()
+    if ex.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during warm-up")
+    clock_path = os.path.join(clock_dir(), f"clocks_rank{rank}.csv")
+    os.makedirs(os.path.dirname(clock_path), exist_ok=True)
+    proc, fh = start_clock_sampler(clock_path, local)
+    time.sleep(0.5)
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        ex.tick(k, v, offsets, frames, out, stream, starts=starts)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    ms = max_over_ranks(e0.elapsed_time(e1), dev)
+    clocks = stop_clock_sampler(proc, fh, clock_path)
+    if ex.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during the timed region")
+    ms_per_step = ms / args.steps
+
+    # end to end: the blocks' frame tokens in from pinned host memory, waypoints back
+    fr_h = frames.cpu().pin_memory()
+    out_h = torch.empty(J, dims.n_waypoints, 2).pin_memory()
+    e2e_steps = max(1, args.steps // 2)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        frames.copy_(fr_h, non_blocking=True)
+        ex.tick(k, v, offsets, frames, out, stream, starts=starts)
+        out_h.copy_(out, non_blocking=True)
+        stream.synchronize()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
+
+    hbm, tensor_tfs, peak_kind = peaks()
+    # each block reads its prefix of the cache at every layer (rows shared by several blocks
+    # count once per block), plus the expert weights once
+    tick_bytes, _ = algorithmic_bytes(dims, prefix, "bf16", weight_bytes)
+    flops = tick_flops(dims, prefix)
+    achieved = tick_bytes / (ms_per_step / 1e3) / 1e9
+    rl_us = max(tick_bytes / (hbm * 1e9), flops / (tensor_tfs * 1e12)) * 1e6
+    line = {
+        "metric": CLIP_METRIC, "value": world * J / (ms_per_step / 1e3), "unit": CLIP_UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_per_step,
+        "us_per_clip": ms_per_step * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f16 (fp32 accumulate)", "data": "synthetic (seeded N(0,1) cache/frames, N(0,1/fan_in) weights)",
+        "config": {"workload": args.workload, "frames": J, "text": c["text"], "delta": c["delta"],
+                   "layers": dims.n_layers, "cache_rows": rows,
+                   "l2": "inputs larger than L2 (the expert weights exceed 129 MB)",
+                   "parallelism": f"replicas x{world}"},
+        "gpu_launches": ex.launches(J) * args.steps,
+        "roofline": {"bound": "hbm", "kernel": "clip tick (whole graph)", "achieved": achieved, "peak": hbm,
+                     "unit": "GB/s", "frac": achieved / hbm, "traffic": None, "peak_source": peak_kind,
+                     "bytes_per_launch": tick_bytes, "launch_us": ms_per_step * 1e3, "flops_per_tick": flops,
+                     "roofline_us": rl_us},
+        "e2e": {"value": world * J * e2e_steps / e2e_s, "unit": CLIP_UNIT,
+                "h2d_bytes_per_step": int(fr_h.numel() * fr_h.element_size()),
+                "d2h_bytes_per_step": int(out_h.numel() * out_h.element_size())},
+        "clocks": clocks,
+    }
+    ex.close()
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def run_reference(args):
     world, rank, _ = dist_env()
     if rank != 0:
@@ -384,6 +541,9 @@ def main():
     from paper_2607_15621_gb300 import synth
     if args.workload in synth.APPEND_WORKLOADS:
         (run_append_reference if args.impl == "reference" else run_append)(args)
+        return
+    if args.workload in synth.CLIP_WORKLOADS:
+        (run_clip_reference if args.impl == "reference" else run_clip)(args)
         return
     if args.impl == "reference":
         run_reference(args)

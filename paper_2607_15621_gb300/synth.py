@@ -72,6 +72,21 @@ class BackboneDims:
 
 BACKBONE = BackboneDims()
 
+# Staleness-masked clip workloads (Sec. 3.2): one clip cache of `text` instruction rows
+# plus `frames` x 4 frame rows; frame j's expert block reads the prefix ending `delta`
+# frames earlier, and all blocks run as one batched tick over explicit row ranges.
+CLIP_WORKLOADS = {
+    "clip_j40_delta1": dict(text=64, frames=40, delta=1, tokens_per_frame=4),
+}
+
+
+def clip_prefixes(workload: str) -> np.ndarray:
+    """Cache rows visible to each frame block of a clip workload (text, plus frames 0 .. j - delta)."""
+    c = CLIP_WORKLOADS[workload]
+    j = np.arange(c["frames"])
+    return np.where(j < c["delta"], c["text"], c["text"] + c["tokens_per_frame"] * (j - c["delta"] + 1)).astype(np.int64)
+
+
 # Cache-append workloads: one call appends n_new tokens for each of `batch`
 # vehicles, each with `length` cached tokens (64 instruction + 40 frames x 4).
 APPEND_WORKLOADS = {

@@ -80,3 +80,16 @@ def test_append_reference_arm_prints_one_line():
     assert line["impl"] == "reference" and line["unit"] == "vehicle-appends/s" and line["value"] > 0
     assert line["config"]["workload"] == "append_b1_l224" and line["config"]["layers"] == 1
     assert line["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_clip_reference_arm_prints_one_line():
+    """The staleness-masked clip workload's reference arm (two expert layers here)."""
+    cmd = [sys.executable, "bench.py", "--impl", "reference", "--workload", "clip_j40_delta1", "--layers", "2",
+           "--steps", "1", "--warmup", "1", "--cpu-seconds", "1"]
+    res = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600)
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [l for l in res.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, res.stdout
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["unit"] == "frame-blocks/s" and line["value"] > 0
+    assert line["config"]["frames"] == 40 and line["config"]["delta"] == 1

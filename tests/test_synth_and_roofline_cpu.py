@@ -101,3 +101,13 @@ def test_tick_roofline_arithmetic():
     assert abs(2 * 42 * per_layer_w * 32 / 1e9 - 28.36) < 0.01
     by32, kv32 = bench.algorithmic_bytes(dims, [96], "fp32", w_bytes)
     assert kv32 == 96 * 32 * 2 * 4096 * 4
+
+
+def test_clip_prefixes_follow_the_visibility_rule():
+    """The clip workload's per-block prefixes are the oracle's visible prefixes (Sec. 3.2)."""
+    from oracle import staleness_oracle
+    c = synth.CLIP_WORKLOADS["clip_j40_delta1"]
+    got = synth.clip_prefixes("clip_j40_delta1")
+    want = [staleness_oracle.visible_prefix(j, c["delta"], c["text"], c["tokens_per_frame"]) for j in range(c["frames"])]
+    assert list(got) == want
+    assert got.max() <= c["text"] + c["tokens_per_frame"] * c["frames"]
