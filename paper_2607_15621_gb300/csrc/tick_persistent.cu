@@ -5,25 +5,36 @@
 // attention head (H clusters, 4H CTAs, one CTA per SM, all co-resident).
 // Every layer runs two phases separated by device-wide counters:
 //   phase A (every cluster = one head h):
-//     x -> RMSNorm (split along K: each CTA normalises its 128 columns and
-//     sends them to the whole cluster) -> the CTA's 96 rows of
-//     [W_q; W_k; W_v] for head h (32 q, 32 k, 32 v dims) on the tensor cores
-//     (tcgen05, accumulator in tensor memory) ->
-//     q, k_ae, v_ae pushed to all 4 CTAs -> Eq. 1 over a quarter of
-//     [K_vlm ; K_ae] per CTA (cache rows staged three 64-key chunks deep in the
-//     shared memory the QKV operands used) -> the 4 fp32 split results merged
-//     (log-sum-exp weights) -> the CTA's 128 output columns of o_h W_o^T
-//     (tcgen05) added into the next residual state with vector atomics
+//     each CTA reads its 128 columns of x, converts them to fp16 and sends them
+//     with the per-token partial sums of x^2 to the whole cluster; four warps
+//     each run the tensor-core MMAs (tcgen05, accumulators in tensor memory) of
+//     one K quarter as soon as that quarter has arrived, for the CTA's 96 rows
+//     of [W_q; W_k; W_v] of head h (32 q, 32 k, 32 v dims; the RMSNorm gain is
+//     folded into the weights and 1/rms is applied to the accumulator sum) ->
+//     q goes to all 4 CTAs, k_ae and v_ae to the CTA that attends over the own
+//     keys -> Eq. 1 over a quarter of [K_vlm ; K_ae] per CTA (cache rows staged
+//     three 64-key chunks deep in the shared memory the QKV operands used) ->
+//     the 4 fp32 split results merged (log-sum-exp weights), each CTA merging
+//     12 rows and sending them to the others -> the CTA's 128 output columns of
+//     o_h W_o^T (tcgen05) added into the next residual state with vector atomics
 //     (cluster 0 also adds the residual itself).
 //   phase B (clusters 0 .. F/64-1; cluster c owns SwiGLU columns 64c..64c+63):
-//     each CTA reads only its 128 columns of x; the per-token sums of x^2 are
-//     completed across the cluster -> RMSNorm of those columns -> the cluster's
-//     128 gate/up rows over this CTA's K quarter (tcgen05) -> the partials
-//     reduce-scattered so that each CTA sums its 16 gate + 16 up rows -> h
-//     pushed to all 4 CTAs -> the CTA's 128 output columns of h W_d^T
-//     (tcgen05) added into the next residual state.
+//     each CTA reads only its 128 columns of x, converts them to fp16 and starts
+//     the cluster's 128 gate/up rows over this K quarter at once, while the
+//     per-token partial sums of x^2 go to the cluster -> the partials are
+//     reduce-scattered so that each CTA sums its 16 gate + 16 up rows, scales
+//     them by 1/rms and forms its 16 SwiGLU columns -> h sent to all 4 CTAs ->
+//     the CTA's 128 output columns of h W_d^T (tcgen05) added into the next
+//     residual state.
 // The residual stream rotates through three fp32 buffers: a phase reads one,
 // accumulates into the next (zeroed one phase earlier) and zeroes the third.
+//
+// Exchanges inside a cluster never use a cluster-wide barrier: a CTA writes
+// into its partners' shared memory with st.async stores that complete on the
+// partner's mbarrier (transaction bytes), and the partner waits on that
+// barrier alone. Each exchange barrier completes once per layer; it is re-armed
+// with the next layer's byte count right after its wait, which always precedes
+// the device-wide counter the senders must pass before sending again.
 //
 // Weights never wait for activations: each CTA's weights are packed in the
 // order it consumes them, as the swizzled K-major images the tensor core reads
@@ -35,7 +46,9 @@
 // 1 of W_d and one empty position; CTAs without SwiGLU work leave positions
 // 8-11 empty), so the QKV images of every layer start at slot 0. The MMAs run
 // with M = 128: the 96-row QKV images are padded with whatever follows them in
-// shared memory, and the accumulator rows that produces are never read.
+// shared memory, and the accumulator rows that produces are never read. Every
+// GEMM is issued by four warps into four accumulators that the epilogue adds:
+// one issuing thread pays a fixed cost per MMA that four issuers overlap.
 #include <cooperative_groups.h>
 #include <math_constants.h>
 
@@ -62,34 +75,34 @@ constexpr int kDS = 128 + 4;           // fp32 row stride of the output transpos
 constexpr int kRowsPerRank = kTokTile / kCl;  // 12
 constexpr int kQkvAtom = 3 * 32 * 128;        // one 64-wide K slice of the CTA's 96 QKV rows (12 KB)
 constexpr int kActAtom = kTokTile * 128;      // one K slice of the 48 token rows (6 KB)
-constexpr uint32_t kTmemCols = 64;            // accumulator: 128 lanes x 48 fp32 columns
+constexpr int kNAcc = 4;                      // accumulators: one per MMA-issuing warp
+constexpr uint32_t kAccCols = 64;             // tensor-memory columns per accumulator (48 used)
+constexpr uint32_t kTmemCols = kNAcc * kAccCols;
 constexpr uint32_t kIdesc = idesc_f16(128, kTokTile);
 constexpr unsigned long long kSpinLimitNs = 1000000000ull;
-#ifndef FSX_NORM_SPLIT
-#define FSX_NORM_SPLIT 1
-#endif
-#ifndef FSX_NORM_BATCH
-#define FSX_NORM_BATCH 2
-#endif
+constexpr int kRecvBytes = kRowsPerRank * kD * 4;  // merge partials one CTA sends another (fp32)
+constexpr int kRsBytes = 32 * kTokTile * 4;        // gate/up partials one CTA sends another (fp32)
+static_assert(kRecvBytes == kRsBytes, "the merge and the gate/up reduce-scatter share the receive buffer");
 
 struct Smem {
   // byte offsets from the 1024-byte aligned base of the dynamic shared memory
-  int bars, lse, ring, act, qbuf, ownk, ownv, tile, recv, recv_lse, total;
+  int bars, gss, rstd, ring, act, qbuf, ownk, ownv, tile, recv, recv_lse, total;
 };
 
 __host__ __device__ inline Smem smem_layout(int d) {
   Smem s{};
-  s.bars = 0;                                  // ring barriers, MMA barrier, TMEM address
-  s.lse = 256;                                 // [48] fp32 log-sum-exp of this split
-  int o = 1024;
+  s.bars = 0;                                  // mbarriers, TMEM address, abort flag
+  s.gss = 512;                                 // [4 ranks][48] fp32 partial sums of x^2
+  s.rstd = 512 + kCl * kTokTile * 4;           // [48] fp32 1 / rms per token
+  int o = 2048;
   s.ring = o;      o += kSlots * kSlotBytes;   // also read 4 KB past its end by the last QKV MMA
-  s.act = o;       o += (d / 64) * kActAtom;   // normalised x, swizzled (B operand of QKV, gate/up)
+  s.act = o;       o += (d / 64) * kActAtom;   // fp16 x, swizzled (B operand of QKV, gate/up)
   s.qbuf = o;      o += kTokTile * kQS * 2;    // q of this head; in phase B the swizzled SwiGLU slice
   s.ownk = o;      o += kTokTile * kQS * 2;    // own keys; later the output transpose
   s.ownv = o;      o += kTokTile * kQS * 2;    // own values
   o = (o + 1023) & ~1023;
-  s.tile = o;      o += 2 * kKeyTile * kD * 2; // fp16 K|V tile; later the merged o_h, swizzled
-  s.recv = o;      o += kCl * kRowsPerRank * kD * 4;  // fp32 split partials of the rows this CTA merges
+  s.tile = o;      o += 2 * kKeyTile * kD * 2; // the merged o_h, swizzled (B operand of W_o)
+  s.recv = o;      o += kCl * kRecvBytes;      // split partials / gate-up partials received
   s.recv_lse = o;  o += kCl * kRowsPerRank * 4;
   s.total = o + 1024;                          // + alignment slack of the dynamic base
   return s;
@@ -116,32 +129,39 @@ __device__ __forceinline__ uint32_t cluster_addr(const void* local, int rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(local)), "r"(rank));
   return r;
 }
-__device__ __forceinline__ void st_cluster_v4(uint32_t addr, uint4 v) {
-  asm volatile("st.shared::cluster.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-               : "memory");
-}
-__device__ __forceinline__ void st_cluster_v2f(uint32_t addr, float a, float b) {
-  asm volatile("st.shared::cluster.v2.f32 [%0], {%1,%2};" ::"r"(addr), "f"(a), "f"(b) : "memory");
-}
-__device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
-  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
-}
 
-// Copy rows x bytes_per_row (multiple of 16) starting at the same local offset to
-// the 3 partner CTAs of the cluster (16-byte remote stores).
-__device__ __forceinline__ void push_rows(const void* base, int rows, int row_stride_bytes, int bytes_per_row,
-                                          int my_rank, int tid, int nthr) {
-  const int upr = bytes_per_row / 16;
-  const unsigned char* b = static_cast<const unsigned char*>(base);
-  for (int i = tid; i < rows * upr * (kPersistCluster - 1); i += nthr) {
-    const int peer_i = i / (rows * upr);
-    const int rest = i - peer_i * rows * upr;
-    const int r = rest / upr;
-    const int u = rest - r * upr;
-    const int peer = peer_i + (peer_i >= my_rank ? 1 : 0);
-    const unsigned char* src = b + static_cast<size_t>(r) * row_stride_bytes + u * 16;
-    st_cluster_v4(cluster_addr(src, peer), *reinterpret_cast<const uint4*>(src));
-  }
+// Arm an exchange barrier (count 1) for its next phase: the arrival plus the
+// bytes the partners will deliver by st.async.
+__device__ __forceinline__ void arm(uint64_t* bar, uint32_t bytes) { mbar_arrive_expect_tx(bar, bytes); }
+
+// tensor memory -> registers: 16 consecutive fp32 columns of each of the four
+// accumulators, added in accumulator order (two loads in flight at a time)
+__device__ __forceinline__ void tmem_ld16_x2(uint32_t taddr, uint32_t (&r)[2][16]) {
+#pragma unroll
+  for (int a = 0; a < 2; ++a)
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[a][0]), "=r"(r[a][1]), "=r"(r[a][2]), "=r"(r[a][3]), "=r"(r[a][4]), "=r"(r[a][5]), "=r"(r[a][6]),
+          "=r"(r[a][7]), "=r"(r[a][8]), "=r"(r[a][9]), "=r"(r[a][10]), "=r"(r[a][11]), "=r"(r[a][12]), "=r"(r[a][13]),
+          "=r"(r[a][14]), "=r"(r[a][15])
+        : "r"(taddr + static_cast<uint32_t>(a) * kAccCols));
+#pragma unroll
+  for (int a = 0; a < 2; ++a)
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[a][0]), "+r"(r[a][1]), "+r"(r[a][2]), "+r"(r[a][3]), "+r"(r[a][4]), "+r"(r[a][5]),
+                   "+r"(r[a][6]), "+r"(r[a][7]), "+r"(r[a][8]), "+r"(r[a][9]), "+r"(r[a][10]), "+r"(r[a][11]),
+                   "+r"(r[a][12]), "+r"(r[a][13]), "+r"(r[a][14]), "+r"(r[a][15])
+                 :
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_ld16_sum4(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[2][16];
+  tmem_ld16_x2(taddr, r);
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[0][i]) + __uint_as_float(r[1][i]);
+  tmem_ld16_x2(taddr + 2 * kAccCols, r);
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = (v[i] + __uint_as_float(r[0][i])) + __uint_as_float(r[1][i]);
 }
 
 // Bounded wait until *counter >= target (one thread polls, the CTA follows).
@@ -171,9 +191,18 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const Smem L = smem_layout(p.d);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bars);
-  uint64_t* mma_bar = full + kSlots;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_bar + 1);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bars);  // [kSlots] weight ring
+  uint64_t* mma_bar = full + kSlots;   // the four issuing warps' MMA groups
+  uint64_t* xbar = mma_bar + 1;        // [4] x quarter + partial sums of x^2 from rank s (phase A)
+  uint64_t* qbar = xbar + kCl;         // q (and own k / v) from the partners
+  uint64_t* rsbar = qbar + 1;          // split partials of the rows this CTA merges
+  uint64_t* agbar = rsbar + 1;         // merged o_h rows of the partners
+  uint64_t* bbar = agbar + 1;          // phase B: partial sums of x^2 and gate/up partials
+  uint64_t* hbar = bbar + 1;           // phase B: the partners' SwiGLU columns
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(hbar + 1);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);  // a wait of this CTA timed out
+  float* gss = reinterpret_cast<float*>(smem + L.gss);
+  float* rstd = reinterpret_cast<float*>(smem + L.rstd);
   unsigned char* ring = smem + L.ring;
   unsigned char* act = smem + L.act;
   __half* qbuf = reinterpret_cast<__half*>(smem + L.qbuf);
@@ -199,7 +228,6 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   const bool in_b = head < p.n_b_clusters;       // phase B participant (whole clusters)
   const int n_b_ctas = p.n_b_clusters * kCl;
   const int total_chunks = p.n_layers * kLayerChunks;
-  volatile int* abort = reinterpret_cast<volatile int*>(smem + L.bars + 96);  // a wait of this CTA timed out
 
   // ---- ring: position q of this CTA's stream uses slot q % kSlots; per layer
   // positions 0-7 are phase-A images, 8-10 phase-B images, the rest empty
@@ -232,18 +260,36 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     if (!ok) *abort = 1;
     return ok;
   };
+  // wait for phase `parity` of an exchange barrier; false after a timeout of this tick
+  auto xwait = [&](uint64_t* bar, int parity) -> bool {
+    if (*abort) return false;
+    const bool ok = mbar_wait_cluster(bar, static_cast<uint32_t>(parity & 1), p.status);
+    if (!ok) *abort = 1;
+    return ok;
+  };
   uint32_t n_mma = 0;  // completed MMA groups (phase of mma_bar)
-  // all threads: wait for the MMA group just committed, then order TMEM reads after it
+  // all threads: wait for the MMA groups just committed, then order TMEM reads after them
   auto wait_mma = [&]() {
     if (*abort == 0 && !mbar_wait(mma_bar, n_mma & 1u, p.status)) *abort = 1;
     ++n_mma;
     tc_fence_after();
   };
 
+  // ---- exchange byte counts, identical in every layer (recomputed at each use from the
+  // launch parameters rather than held in registers across the attention)
+#define FSX_T (p.n_action + p.n_frame)
+#define FSX_X_BYTES static_cast<uint32_t>(FSX_T * (128 * 2 + 4))  // fp16 x quarter + partial sums, per partner
+#define FSX_RS_BYTES static_cast<uint32_t>((kCl - 1) * (kRecvBytes + kRowsPerRank * 4))
+#define FSX_AG_BYTES static_cast<uint32_t>((kCl - 1) * kRowsPerRank * kD * 2)
+#define FSX_B_BYTES static_cast<uint32_t>((kCl - 1) * (kRsBytes + FSX_T * 4))
+#define FSX_H_BYTES static_cast<uint32_t>((kCl - 1) * FSX_T * 32)
+#define FSX_Q_BYTES static_cast<uint32_t>((kCl - 1) * FSX_T * 64 * (rank == own_rank ? 3 : 1))
+
   if (tid == 0) {
     *abort = 0;
     for (int i = 0; i < kSlots; ++i) mbar_init(full + i, 1);
-    mbar_init(mma_bar, 1);
+    mbar_init(mma_bar, kNAcc);
+    for (int i = 0; i < kCl + 5; ++i) mbar_init(xbar + i, 1);
     for (int q = 0; q < kSlots; ++q) issue(q);
   }
 
@@ -255,7 +301,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   if (!bad && o_hi > o_lo)  // a non-empty cache needs every layer's rows
     for (int l = 0; l < p.n_layers; ++l)
       bad = bad || p.targs->k_cache[l] == nullptr || p.targs->v_cache[l] == nullptr;
-  __syncthreads();
+  cluster.sync();  // barrier initialisation visible to the partners before any st.async
   if (bad) {
     if (cta == 0 && tid == 0) set_status(p.status, kStatusDeviceArg);
     if (tid == 0)
@@ -263,14 +309,14 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     return;
   }
 
-  // ---- tensor memory for the accumulator (one CTA per SM: never contended)
+  // ---- tensor memory for the four accumulators (one CTA per SM: never contended)
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(tmem_slot)),
                  "r"(kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  // token rows T..47 of the activation image stay zero for the whole tick
+  // token rows T..47 of the activation image start at zero
   for (int i = tid; i < (kTokTile - T) * (d / 8); i += kThr) {
     const int r = T + i / (d / 8);
     const int k = (i % (d / 8)) * 8;
@@ -282,6 +328,13 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(tmem_slot);
   const uint32_t ring_a = smem_addr(ring);
   const uint32_t act_a = smem_addr(act);
+  // one MMA-issuing warp: K steps kk0 .. kk0 + nk - 1 (K = 16 each) of one 64-wide K
+  // slice into accumulator `acc`: D[128 x 48] (+)= A[128 rows] . B[48 tokens]^T
+  auto mma_k = [&](int acc, uint32_t a_addr, uint32_t b_addr, int kk0, int nk, bool first) {
+    for (int kk = kk0; kk < kk0 + nk; ++kk)
+      umma_f16(tmem + static_cast<uint32_t>(acc) * kAccCols, sw128_desc(a_addr + kk * 32),
+               sw128_desc(b_addr + kk * 32), kIdesc, (first && kk == kk0) ? 0u : 1u);
+  };
 
   const long long Lc = o_hi - o_lo;
 
@@ -308,135 +361,88 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       __stcg(X0 + xs + e, 0.f);
     }
   }
-  arrive(p.counters + 0);
 
-  // x (state buffer in L2) -> RMSNorm -> fp16 rows of the swizzled activation
-  // image. Warp w takes rows w, w+8, ... (rotated by 8 (cta mod 6), so that the
-  // 128 CTAs reading the same 84 KB spread over all rows at any moment instead of
-  // queueing on the same L2 lines); lane l takes columns 16l..16l+15. Every load
-  // of the warp is issued before the first use: one L2 round trip covers all.
-  const int row_rot = (cta % 6) * 8;
-  auto load_normalized = [&](const float* Xs) {
-    constexpr int kRowsPerWarp = kTokTile / (kThr / 32);  // 6
-    constexpr int kBatch = FSX_NORM_BATCH;                // rows in flight per warp
-#pragma unroll 1
-    for (int i0 = 0; i0 < kRowsPerWarp; i0 += kBatch) {
-      float4 v[kBatch][4];
+  // This thread's share of a CTA's 128 columns of x when they are converted to fp16:
+  // 8-column unit xu of rows xr0, xr0 + 16, xr0 + 32.
+  const int xu = tid & 15;
+  const int xr0 = tid >> 4;
+  // fp32 columns of this thread's rows -> fp16 x image (local, and the partners when
+  // `send_x`), per-token partial sums of x^2 -> gss[rank] here and in the partners;
+  // the partners' `peer_bar` counts the bytes
+  auto load_quarter = [&](const float* Xs, int col0, int k0, bool send_x, uint64_t* peer_bar) {
 #pragma unroll
-      for (int i = 0; i < kBatch; ++i) {
-        const int r = (warp + 8 * (i0 + i) + row_rot) % kTokTile;
-        if (r < T) {
-          const float* xr = Xs + static_cast<size_t>(r) * d + lane * 16;
-#pragma unroll
-          for (int j = 0; j < 4; ++j) v[i][j] = ld_cg4(xr + 4 * j);
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < kBatch; ++i) {
-        const int r = (warp + 8 * (i0 + i) + row_rot) % kTokTile;
-        if (r < T) {
-          float ss = 0.f;
-#pragma unroll
-          for (int j = 0; j < 4; ++j) ss += v[i][j].x * v[i][j].x + v[i][j].y * v[i][j].y + v[i][j].z * v[i][j].z + v[i][j].w * v[i][j].w;
-          ss = warp_sum(ss);
-          const float rstd = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
-          uint4 lo, hi;
-          lo.x = pack_half2(v[i][0].x * rstd, v[i][0].y * rstd);
-          lo.y = pack_half2(v[i][0].z * rstd, v[i][0].w * rstd);
-          lo.z = pack_half2(v[i][1].x * rstd, v[i][1].y * rstd);
-          lo.w = pack_half2(v[i][1].z * rstd, v[i][1].w * rstd);
-          hi.x = pack_half2(v[i][2].x * rstd, v[i][2].y * rstd);
-          hi.y = pack_half2(v[i][2].z * rstd, v[i][2].w * rstd);
-          hi.z = pack_half2(v[i][3].x * rstd, v[i][3].y * rstd);
-          hi.w = pack_half2(v[i][3].z * rstd, v[i][3].w * rstd);
-          *reinterpret_cast<uint4*>(act + sw128_offset(kTokTile, r, lane * 16)) = lo;
-          *reinterpret_cast<uint4*>(act + sw128_offset(kTokTile, r, lane * 16 + 8)) = hi;
-        }
-      }
-    }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // visible to the tensor core
-    __syncthreads();
-  };
-
-  // RMSNorm split along K inside the cluster (phase A): this rank reads only its 128
-  // columns of x, sends its per-token partial sums of x^2 to every rank, normalises its
-  // columns and writes them into the activation image of all four ranks, so each CTA
-  // holds the full [48 x 512] fp16 image for its QKV rows. gss lives in dstT, idle
-  // from the end of the previous phase B to the W_o transpose.
-  auto load_normalized_split = [&](const float* Xs) {
-    float* gss = dstT;  // [4 ranks][48]
-    constexpr int kRowsPerWarp = kTokTile / (kThr / 32);  // 6
-    float4 xv[kRowsPerWarp];
-#pragma unroll
-    for (int i = 0; i < kRowsPerWarp; ++i) {
-      const int r = warp + 8 * i;
-      xv[i] = r < T ? ld_cg4(Xs + static_cast<size_t>(r) * d + rank * 128 + lane * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-#pragma unroll
-    for (int i = 0; i < kRowsPerWarp; ++i) {
-      const int r = warp + 8 * i;
-      const float ps = warp_sum(xv[i].x * xv[i].x + xv[i].y * xv[i].y + xv[i].z * xv[i].z + xv[i].w * xv[i].w);
-      if (r < T && lane < kCl) st_cluster_f32(cluster_addr(gss + rank * kTokTile + r, lane), ps);
-    }
-    cluster.sync();  // every rank's partial sums arrived
-#pragma unroll
-    for (int i = 0; i < kRowsPerWarp; ++i) {
-      const int r = warp + 8 * i;
+    for (int i = 0; i < 3; ++i) {
+      const int r = xr0 + 16 * i;
+      float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
       if (r < T) {
-        const float ss = ((gss[r] + gss[kTokTile + r]) + gss[2 * kTokTile + r]) + gss[3 * kTokTile + r];
-        const float rstd = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
-        const float lo = __uint_as_float(pack_half2(xv[i].x * rstd, xv[i].y * rstd));
-        const float hi = __uint_as_float(pack_half2(xv[i].z * rstd, xv[i].w * rstd));
-        unsigned char* dst = act + sw128_offset(kTokTile, r, rank * 128 + lane * 4);
+        a = ld_cg4(Xs + static_cast<size_t>(r) * d + col0 + xu * 8);
+        b = ld_cg4(Xs + static_cast<size_t>(r) * d + col0 + xu * 8 + 4);
+      }
+      float ss = a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w + b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
 #pragma unroll
-        for (int peer = 0; peer < kCl; ++peer) st_cluster_v2f(cluster_addr(dst, peer), lo, hi);
+      for (int o = 8; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);  // the row's 16 threads
+      if (r < T && *abort == 0) {
+        const uint4 h = make_uint4(pack_half2(a.x, a.y), pack_half2(a.z, a.w), pack_half2(b.x, b.y), pack_half2(b.z, b.w));
+        unsigned char* dst = act + sw128_offset(kTokTile, r, k0 + xu * 8);
+        *reinterpret_cast<uint4*>(dst) = h;
+        if (xu == 0) gss[rank * kTokTile + r] = ss;
+#pragma unroll
+        for (int pi = 1; pi < kCl; ++pi) {
+          const int peer = (rank + pi) & (kCl - 1);
+          const uint32_t pb = cluster_addr(peer_bar, peer);
+          if (send_x) st_async_v4(cluster_addr(dst, peer), h, pb);
+          if (xu == 0) st_async_b32(cluster_addr(gss + rank * kTokTile + r, peer), __float_as_uint(ss), pb);
+        }
       }
     }
-    asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
-    cluster.sync();  // the full image is in every rank
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // visible to the tensor core
   };
-
-  // add the CTA's [48 x 128] transposed output (dstT) into X_next columns col0..col0+127,
-  // plus the residual X_cur when this is cluster 0
-  auto scatter_add = [&](float* Xn, const float* Xc, int col0, bool add_residual) {
-    for (int i = tid; i < T * 32; i += kThr) {
-      const int t = i >> 5;
-      const int c4 = (i & 31) * 4;
-      float4 v = *reinterpret_cast<const float4*>(dstT + t * kDS + c4);
-      if (add_residual) {
-        const float4 r = ld_cg4(Xc + static_cast<size_t>(t) * d + col0 + c4);
-        v.x += r.x;
-        v.y += r.y;
-        v.z += r.z;
-        v.w += r.w;
-      }
-      red_add_v4(Xn + static_cast<size_t>(t) * d + col0 + c4, v);
+  // 1 / rms of every token from the four ranks' partial sums (rank order)
+  auto compute_rstd = [&]() {
+    if (tid < T) {
+      const float ss = ((gss[tid] + gss[kTokTile + tid]) + gss[2 * kTokTile + tid]) + gss[3 * kTokTile + tid];
+      rstd[tid] = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
     }
   };
-
-  // accumulator (128 output columns x 48 tokens) -> dstT[token][column]; warps
-  // 0-3 take tokens 0-31, warps 4-7 tokens 32-47 of their 32 TMEM lanes
+  // a CTA's [48 x 128] transposed output (dstT) added into X_next columns col0..col0+127,
+  // plus the residual `res` when given: warp w takes rows w, w + 8, ..., lane l columns
+  // 4l..4l+3, so every vector atomic of a warp covers one contiguous 512-byte row
+  auto scatter_add = [&](float* Xn, int col0, const float4 (&res)[6], bool add_residual) {
+#pragma unroll
+    for (int i = 0; i < 6; ++i) {
+      const int t = warp + 8 * i;
+      if (t < T) {
+        float4 v = *reinterpret_cast<const float4*>(dstT + t * kDS + lane * 4);
+        if (add_residual) {
+          v.x += res[i].x;
+          v.y += res[i].y;
+          v.z += res[i].z;
+          v.w += res[i].w;
+        }
+        red_add_v4(Xn + static_cast<size_t>(t) * d + col0 + lane * 4, v);
+      }
+    }
+  };
+  auto load_residual = [&](const float* Xs, int col0, float4 (&res)[6]) {
+#pragma unroll
+    for (int i = 0; i < 6; ++i) {
+      const int t = warp + 8 * i;
+      res[i] = t < T ? ld_cg4(Xs + static_cast<size_t>(t) * d + col0 + lane * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  };
+  // the four accumulators' sum (128 output columns x 48 tokens) -> dstT[token][column];
+  // warps 0-3 take tokens 0-31, warps 4-7 tokens 32-47 of their 32 TMEM lanes
   auto tmem_to_dstT = [&]() {
     const int col = (warp & 3) * 32 + lane;
     const uint32_t taddr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
     for (int c0 = warp < 4 ? 0 : 32; c0 < (warp < 4 ? 32 : 48); c0 += 16) {
       float v[16];
       __syncwarp();
-      tmem_ld16(taddr + static_cast<uint32_t>(c0), v);
+      tmem_ld16_sum4(taddr + static_cast<uint32_t>(c0), v);
 #pragma unroll
       for (int j = 0; j < 16; ++j) dstT[(c0 + j) * kDS + col] = v[j];
     }
     tc_fence_before();
     __syncthreads();
-  };
-
-  // one K slice (4 MMAs of K = 16) of D[128 x 48] (+)= A[128 rows] . B[48 tokens]^T
-  auto mma_slice = [&](uint32_t a_addr, uint32_t b_addr, bool first) {
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk)
-      umma_f16(tmem, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32), kIdesc,
-               (first && kk == 0) ? 0u : 1u);
   };
 
   // ---- this CTA's cache rows of a layer, staged in the shared memory that is idle
@@ -514,23 +520,29 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     const int n = min(kStageKeys, n_cache - j * kStageKeys);
     unsigned char* kb = stage_base + (j % kNB) * kBufBytes;
     if (sizeof(CT) == 2) {
-      uint4 v[kCvtIters];
+      // two rounds of half the units, every load of a round before its first store
+      constexpr int kHalf = (kCvtIters + 1) / 2;
 #pragma unroll
-      for (int it = 0; it < kCvtIters; ++it) {  // every load before the first store
-        const int i = tid + it * kThr;
-        const int r = i >> 4;
-        const int key = r >= kStageKeys ? r - kStageKeys : r;
-        if (r < 2 * kStageKeys && key < n) v[it] = *reinterpret_cast<const uint4*>(kb + r * kRowStride + (i & 15) * 16);
-      }
+      for (int r0 = 0; r0 < kCvtIters; r0 += kHalf) {
+        uint4 v[kHalf];
 #pragma unroll
-      for (int it = 0; it < kCvtIters; ++it) {
-        const int i = tid + it * kThr;
-        const int r = i >> 4;
-        const int key = r >= kStageKeys ? r - kStageKeys : r;
-        if (r < 2 * kStageKeys && key < n)
-          *reinterpret_cast<uint4*>(kb + r * kRowStride + (i & 15) * 16) =
-              make_uint4(bf16x2_to_half2(v[it].x), bf16x2_to_half2(v[it].y), bf16x2_to_half2(v[it].z),
-                         bf16x2_to_half2(v[it].w));
+        for (int it = 0; it < kHalf; ++it) {
+          const int i = tid + (r0 + it) * kThr;
+          const int r = i >> 4;
+          const int key = r >= kStageKeys ? r - kStageKeys : r;
+          if (r0 + it < kCvtIters && r < 2 * kStageKeys && key < n)
+            v[it] = *reinterpret_cast<const uint4*>(kb + r * kRowStride + (i & 15) * 16);
+        }
+#pragma unroll
+        for (int it = 0; it < kHalf; ++it) {
+          const int i = tid + (r0 + it) * kThr;
+          const int r = i >> 4;
+          const int key = r >= kStageKeys ? r - kStageKeys : r;
+          if (r0 + it < kCvtIters && r < 2 * kStageKeys && key < n)
+            *reinterpret_cast<uint4*>(kb + r * kRowStride + (i & 15) * 16) =
+                make_uint4(bf16x2_to_half2(v[it].x), bf16x2_to_half2(v[it].y), bf16x2_to_half2(v[it].z),
+                           bf16x2_to_half2(v[it].w));
+        }
       }
     } else {
       // 32-byte fp32 unit u of a row -> 16-byte fp16 unit u at the row start. A row's 16
@@ -558,10 +570,25 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     __syncthreads();
   };
 
+  // ---- arm the exchange barriers for layer 0, then publish the token assembly
+  if (tid < kTokTile) rstd[tid] = 0.f;  // padding tokens T..47 stay at zero
+  if (tid == 0) {
+    for (int s_ = 1; s_ < kCl; ++s_) arm(xbar + ((rank + s_) & (kCl - 1)), FSX_X_BYTES);
+    arm(qbar, FSX_Q_BYTES);
+    arm(rsbar, FSX_RS_BYTES);
+    arm(agbar, FSX_AG_BYTES);
+    if (in_b) {
+      arm(bbar, FSX_B_BYTES);
+      arm(hbar, FSX_H_BYTES);
+    }
+  }
+  arrive(p.counters + 0);
+
   int q0 = 0;  // first ring position of the current layer
   const float scale_log2 = 1.4426950408889634f * rsqrtf(static_cast<float>(kD));
 
   for (int layer = 0; layer < p.n_layers; ++layer, q0 += kLayerChunks) {
+    const int par = layer & 1;  // phase of every exchange barrier in this layer
     const int sA = 2 * layer;
     float* Xc = X0 + static_cast<size_t>(sA % 3) * xs;        // layer input
     float* Xm = X0 + static_cast<size_t>((sA + 1) % 3) * xs;  // after attention
@@ -578,53 +605,82 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       const int e1 = static_cast<int>(static_cast<long long>(n_elem) * (cta + 1) / G);
       for (int e = e0 + tid; e < e1; e += kThr) __stcg(Xz + e, 0.f);
     }
-#if FSX_NORM_SPLIT
-    load_normalized_split(Xc);
-#else
-    load_normalized(Xc);
-#endif
+    // this rank's 128 columns of x -> fp16 image here and in the partners (K slices
+    // 2 rank, 2 rank + 1), partial sums of x^2 to every rank
+    load_quarter(Xc, rank * 128, rank * 128, true, xbar + rank);
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the local quarter -> tensor core
+    __syncthreads();
 
-    // --- QKV: D[96 (+32 unused) rows x 48 tokens] over K = 512; the 12 KB K
-    // slices lie back to back in slots 0-5, so slice a needs the slots it touches
-    if (warp == 0) {
+    // --- QKV: D[96 (+32 unused) rows x 48 tokens] over K = 512. Warp w < 4 runs K quarter w
+    // (slices 2w, 2w + 1: rank w's columns of x) into accumulator w as soon as rank w's
+    // columns and the weight slots under them have arrived; the 12 KB K slices lie back
+    // to back in slots 0-5
+    if (warp < kNAcc) {
       tc_fence_after();
+      const int a0 = 2 * warp;
       bool ok = true;
-      int waited = -1;
-      for (int a = 0; a < d / 64; ++a) {
-        const int last = (a * kQkvAtom + kQkvAtom - 1) / kSlotBytes;
-        while (waited < last) ok = wait_chunk(q0 + ++waited) && ok;
-        if (ok && lane == 0) mma_slice(ring_a + a * kQkvAtom, act_a + a * kActAtom, a == 0);
-        __syncwarp();
+      for (int sl = (a0 * kQkvAtom) / kSlotBytes; sl <= ((a0 + 2) * kQkvAtom - 1) / kSlotBytes; ++sl)
+        ok = wait_chunk(q0 + sl) && ok;
+      if (warp != rank) ok = xwait(xbar + warp, par) && ok;
+      if (ok && lane == 0) {
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the partner's columns -> tensor core
+        mma_k(warp, ring_a + a0 * kQkvAtom, act_a + a0 * kActAtom, 0, 4, true);
+        mma_k(warp, ring_a + (a0 + 1) * kQkvAtom, act_a + (a0 + 1) * kActAtom, 0, 4, false);
       }
+      __syncwarp();
       if (lane == 0) umma_commit(mma_bar);
       __syncwarp();
     }
+    // every partner's partial sums of x^2 have arrived: 1 / rms per token; re-arm for the next layer
+    for (int s_ = 1; s_ < kCl; ++s_) xwait(xbar + ((rank + s_) & (kCl - 1)), par);
+    if (tid == 0 && *abort == 0)
+      for (int s_ = 1; s_ < kCl; ++s_) arm(xbar + ((rank + s_) & (kCl - 1)), FSX_X_BYTES);
+    compute_rstd();
+    __syncthreads();
     wait_mma();
     for (int j = 0; j < kNB && j < n_chunks; ++j)  // slots 2-5 and the activation image are free
       stage_issue(j, kc, vc);
-    // rows 32j..32j+31 of the accumulator are q, k, v dims 32 rank .. 32 rank + 31
+    // rows 32j..32j+31 of the accumulators are q, k, v dims 32 rank .. 32 rank + 31,
+    // scaled by 1 / rms of their token
     if ((warp & 3) < 3) {
       const int kind = warp & 3;
       __half* b = kind == 0 ? qbuf : (kind == 1 ? ownk : ownv);
       const int dim = rank * 32 + lane;
       const uint32_t taddr = tmem + (static_cast<uint32_t>(kind * 32) << 16);
-      for (int c0 = warp < 4 ? 0 : 32; c0 < (warp < 4 ? 32 : 48); c0 += 16) {
+      const int c_lo = warp < 4 ? 0 : 32;
+      const int c_hi = warp < 4 ? 32 : 48;
+      for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
         float v[16];
         __syncwarp();
-        tmem_ld16(taddr + static_cast<uint32_t>(c0), v);
+        tmem_ld16_sum4(taddr + static_cast<uint32_t>(c0), v);
 #pragma unroll
-        for (int j = 0; j < 16; ++j) b[(c0 + j) * kQS + dim] = __float2half_rn(v[j]);
+        for (int j = 0; j < 16; ++j) b[(c0 + j) * kQS + dim] = __float2half_rn(v[j] * rstd[c0 + j]);
+      }
+      __syncwarp();
+      // this warp's token rows below T (dims 32 rank .. + 31, four 16-byte units a row): q to
+      // every partner, own k and v to the rank that attends over the own keys
+      if (*abort == 0 && (kind == 0 || own_rank != rank)) {
+        for (int i = lane; i < (min(c_hi, T) - c_lo) * 4; i += 32) {
+          const __half* src = b + (c_lo + (i >> 2)) * kQS + rank * 32 + (i & 3) * 8;
+          const uint4 v = *reinterpret_cast<const uint4*>(src);
+          if (kind == 0) {
+#pragma unroll
+            for (int pi = 1; pi < kCl; ++pi) {
+              const int peer = (rank + pi) & (kCl - 1);
+              st_async_v4(cluster_addr(src, peer), v, cluster_addr(qbar, peer));
+            }
+          } else {
+            st_async_v4(cluster_addr(src, own_rank), v, cluster_addr(qbar, own_rank));
+          }
+        }
       }
     }
     tc_fence_before();
     __syncthreads();
     if (tid == 0)  // slots 0, 1 are free: W_o of this layer (slots 2-5 stage the cache)
       for (int i = kSlots; i < kPersistAChunks; ++i) issue(q0 + i);
-    // this rank's 32 dims of q, k_ae, v_ae (48 rows x 64 bytes each) to the partners
-    push_rows(qbuf + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
-    push_rows(ownk + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
-    push_rows(ownv + rank * 32, kTokTile, kQS * 2, 64, rank, tid, kThr);
-    cluster.sync();  // q, own k, own v complete in every CTA
+    xwait(qbar, par);  // q (and on the own-key rank, own k / v) of every partner
+    if (tid == 0 && *abort == 0) arm(qbar, FSX_Q_BYTES);
 
     // --- Eq. 1 over this CTA's cache keys, then its own keys, in 32-key tiles. Warp w < 6
     // takes query rows 16 (w % 3) .. +15 and every other key tile (tiles kh, kh + 2, ...
@@ -786,8 +842,20 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     }
 
     // --- merge the 4 splits: every row's normalised fp32 partial and log-sum-exp go
-    // straight from the registers to the rank that owns the row
-    if (warp < 6) {
+    // straight from the registers to the rank that owns the row (st.async to the partners)
+    if (warp < 6 && *abort == 0) {
+      auto put2 = [&](float* ptr, int dst, float a, float b) {
+        if (dst == rank)
+          *reinterpret_cast<float2*>(ptr) = make_float2(a, b);
+        else
+          st_async_v2(cluster_addr(ptr, dst), __float_as_uint(a), __float_as_uint(b), cluster_addr(rsbar, dst));
+      };
+      auto put1 = [&](float* ptr, int dst, float a) {
+        if (dst == rank)
+          *ptr = a;
+        else
+          st_async_b32(cluster_addr(ptr, dst), __float_as_uint(a), cluster_addr(rsbar, dst));
+      };
       const int qr0 = qt * 16 + (lane >> 2);
       const int qr1 = qr0 + 8;
       const int own0 = qr0 / kRowsPerRank;
@@ -799,18 +867,20 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
 #pragma unroll
       for (int nb = 0; nb < 8; ++nb) {
         const int c = kh * 64 + nb * 8 + 2 * (lane & 3);
-        st_cluster_v2f(cluster_addr(d0 + c, own0), o_fin[nb][0] * inv0, o_fin[nb][1] * inv0);
-        st_cluster_v2f(cluster_addr(d1 + c, own1), o_fin[nb][2] * inv1, o_fin[nb][3] * inv1);
+        put2(d0 + c, own0, o_fin[nb][0] * inv0, o_fin[nb][1] * inv0);
+        put2(d1 + c, own1, o_fin[nb][2] * inv1, o_fin[nb][3] * inv1);
       }
       if (kh == 0 && (lane & 3) == 0) {
-        st_cluster_f32(cluster_addr(recv_lse + rank * kRowsPerRank + qr0 - own0 * kRowsPerRank, own0),
-                       l_run[0] > 0.f ? m_run[0] + log2f(l_run[0]) : -CUDART_INF_F);
-        st_cluster_f32(cluster_addr(recv_lse + rank * kRowsPerRank + qr1 - own1 * kRowsPerRank, own1),
-                       l_run[1] > 0.f ? m_run[1] + log2f(l_run[1]) : -CUDART_INF_F);
+        put1(recv_lse + rank * kRowsPerRank + qr0 - own0 * kRowsPerRank, own0,
+             l_run[0] > 0.f ? m_run[0] + log2f(l_run[0]) : -CUDART_INF_F);
+        put1(recv_lse + rank * kRowsPerRank + qr1 - own1 * kRowsPerRank, own1,
+             l_run[1] > 0.f ? m_run[1] + log2f(l_run[1]) : -CUDART_INF_F);
       }
     }
-    cluster.sync();
-    // merged rows of o_h -> swizzled image in every partner's obuf (the W_o B operand)
+    xwait(rsbar, par);  // every partner's partials of the rows this CTA merges
+    __syncthreads();    // and this CTA's own
+    if (tid == 0 && *abort == 0) arm(rsbar, FSX_RS_BYTES);
+    // merged rows of o_h -> swizzled image (the W_o B operand) here and in every partner
     {
       const int r0 = rank * kRowsPerRank;
       for (int i = tid; i < kRowsPerRank * (kD / 4); i += kThr) {
@@ -837,43 +907,44 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         uint2 out;
         out.x = pack_half2(a0 * inv, a1 * inv);
         out.y = pack_half2(a2 * inv, a3 * inv);
-        *reinterpret_cast<uint2*>(obuf + sw128_offset(kTokTile, row, c)) = out;
+        unsigned char* dst = obuf + sw128_offset(kTokTile, row, c);
+        *reinterpret_cast<uint2*>(dst) = out;
+        if (*abort == 0) {
+#pragma unroll
+          for (int pi = 1; pi < kCl; ++pi) {
+            const int peer = (rank + pi) & (kCl - 1);
+            st_async_v2(cluster_addr(dst, peer), out.x, out.y, cluster_addr(agbar, peer));
+          }
+        }
         if (p.attn_capture != nullptr && row < T)
           *reinterpret_cast<uint2*>(p.attn_capture + (static_cast<size_t>(layer) * T + row) * HD + head * kD + c) = out;
       }
     }
+    xwait(agbar, par);  // the partners' merged rows
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // o_h -> tensor core
     __syncthreads();
-    for (int i = tid; i < kRowsPerRank * (kD / 8) * (kCl - 1); i += kThr) {
-      const int peer_i = i / (kRowsPerRank * (kD / 8));
-      const int rest = i - peer_i * kRowsPerRank * (kD / 8);
-      const int row = rank * kRowsPerRank + rest / (kD / 8);
-      const int u = rest % (kD / 8);
-      const int peer = peer_i + (peer_i >= rank ? 1 : 0);
-      const uint32_t off = sw128_offset(kTokTile, row, u * 8);
-      st_cluster_v4(cluster_addr(obuf + off, peer), *reinterpret_cast<const uint4*>(obuf + off));
-    }
-    asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
-    cluster.sync();  // o_h complete everywhere; ownk/ownv free for the transpose
+    if (tid == 0 && *abort == 0) arm(agbar, FSX_AG_BYTES);
 
-    // --- W_o: this CTA's 128 output columns for head h, K = 128 (slots 0, 1)
-    if (warp == 0) {
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    // --- W_o: this CTA's 128 output columns for head h, K = 128 (slots 0, 1); warp w:
+    // slice w / 2, K steps 2 (w % 2) .. + 1
+    if (warp < kNAcc) {
       tc_fence_after();
-      for (int a = 0; a < 2; ++a) {
-        const bool ok = wait_chunk(q0 + kSlots + a);
-        if (ok && lane == 0) mma_slice(ring_a + a * kSlotBytes, smem_addr(obuf) + a * kActAtom, a == 0);
-        __syncwarp();
-      }
+      const int a = warp >> 1;
+      const bool ok = wait_chunk(q0 + kSlots + a);
+      if (ok && lane == 0) mma_k(warp, ring_a + a * kSlotBytes, smem_addr(obuf) + a * kActAtom, (warp & 1) * 2, 2, true);
+      __syncwarp();
       if (lane == 0) umma_commit(mma_bar);
       __syncwarp();
     }
+    float4 res[6];
+    if (head == 0) load_residual(Xc, rank * 128, res);  // cluster 0 adds the residual itself
     wait_mma();
     tmem_to_dstT();
     if (tid == 0) {  // slots 0, 1 free (all of 0-5 for CTAs without phase B): next layer's QKV
       const int n = in_b ? 2 : kSlots;
       for (int i = 0; i < n; ++i) issue(q0 + kLayerChunks + i);
     }
-    scatter_add(Xm, Xc, rank * 128, head == 0);
+    scatter_add(Xm, rank * 128, res, head == 0);
     arrive(p.counters + sA + 1);
 
     // =========================== phase B ===========================
@@ -885,53 +956,26 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         const int e1 = static_cast<int>(static_cast<long long>(n_elem) * (cta + 1) / n_b_ctas);
         for (int e = e0 + tid; e < e1; e += kThr) __stcg(Xc + e, 0.f);
       }
-      // --- RMSNorm split along K: this rank reads only its 128 columns of x, sends its
-      // per-token partial sums of x^2 to every CTA of the cluster, and normalises its
-      // columns into the first two K slices of the activation image
-      float* gss = dstT;  // [4 ranks][48] partial sums of x^2 (dstT is idle until W_d)
-      constexpr int kRowsPerWarp = kTokTile / (kThr / 32);  // 6
-      float4 xv[kRowsPerWarp];
-#pragma unroll
-      for (int i = 0; i < kRowsPerWarp; ++i) {
-        const int r = warp + 8 * i;
-        xv[i] = r < T ? ld_cg4(Xm + static_cast<size_t>(r) * d + rank * 128 + lane * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-#pragma unroll
-      for (int i = 0; i < kRowsPerWarp; ++i) {
-        const int r = warp + 8 * i;
-        const float ps = warp_sum(xv[i].x * xv[i].x + xv[i].y * xv[i].y + xv[i].z * xv[i].z + xv[i].w * xv[i].w);
-        if (r < T && lane < kCl) st_cluster_f32(cluster_addr(gss + rank * kTokTile + r, lane), ps);
-      }
-      cluster.sync();  // every rank's partial sums arrived
-#pragma unroll
-      for (int i = 0; i < kRowsPerWarp; ++i) {
-        const int r = warp + 8 * i;
-        if (r < T) {
-          const float ss = ((gss[r] + gss[kTokTile + r]) + gss[2 * kTokTile + r]) + gss[3 * kTokTile + r];
-          const float rstd = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
-          uint2 pk;
-          pk.x = pack_half2(xv[i].x * rstd, xv[i].y * rstd);
-          pk.y = pack_half2(xv[i].z * rstd, xv[i].w * rstd);
-          *reinterpret_cast<uint2*>(act + sw128_offset(kTokTile, r, lane * 4)) = pk;
-        }
-      }
+      // this rank's 128 columns of x -> fp16 K slices 0, 1 here (no exchange: each CTA runs
+      // the gate/up MMAs over its own K quarter), partial sums of x^2 to every rank
+      load_quarter(Xm, rank * 128, 0, false, bbar);
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // visible to the tensor core
       __syncthreads();
-      // gate/up over this rank's K quarter: D[128 rows x 48 tokens], rows 32s..32s+31 =
-      // the 16 gate and 16 up rows of rank s's SwiGLU columns (K slices in slots 2, 3)
-      if (warp == 0) {
+      // gate/up over this rank's K quarter: D[128 rows x 48 tokens], rows 32s..32s+31 = the
+      // 16 gate and 16 up rows of rank s's SwiGLU columns (K slices in slots 2, 3); warp w:
+      // slice w / 2, K steps 2 (w % 2) .. + 1
+      if (warp < kNAcc) {
         tc_fence_after();
-        for (int a = 0; a < 2; ++a) {
-          const bool ok = wait_chunk(q0 + kPersistAChunks + a);
-          if (ok && lane == 0) mma_slice(ring_a + (2 + a) * kSlotBytes, act_a + a * kActAtom, a == 0);
-          __syncwarp();
-        }
+        const int a = warp >> 1;
+        const bool ok = wait_chunk(q0 + kPersistAChunks + a);
+        if (ok && lane == 0) mma_k(warp, ring_a + (2 + a) * kSlotBytes, act_a + a * kActAtom, (warp & 1) * 2, 2, true);
+        __syncwarp();
         if (lane == 0) umma_commit(mma_bar);
         __syncwarp();
       }
       wait_mma();
-      // reduce-scatter of the K partials: rows 32s..32s+31 go to rank s as
-      // recv[this rank][row][48 tokens] (fp32)
+      // reduce-scatter of the K partials: rows 32q..32q+31 (the accumulators' sum) go to rank q
+      // as recv[this rank][row][48 tokens] (fp32)
       {
         const int q = warp & 3;
         const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16);
@@ -939,61 +983,84 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         for (int c0 = warp < 4 ? 0 : 32; c0 < (warp < 4 ? 32 : 48); c0 += 16) {
           float v[16];
           __syncwarp();
-          tmem_ld16(taddr + static_cast<uint32_t>(c0), v);
+          tmem_ld16_sum4(taddr + static_cast<uint32_t>(c0), v);
 #pragma unroll
-          for (int j = 0; j < 16; j += 4)
-            st_cluster_v4(cluster_addr(dst + c0 + j, q),
-                          make_uint4(__float_as_uint(v[j]), __float_as_uint(v[j + 1]), __float_as_uint(v[j + 2]),
-                                     __float_as_uint(v[j + 3])));
+          for (int j = 0; j < 16; j += 4) {
+            const uint4 u = make_uint4(__float_as_uint(v[j]), __float_as_uint(v[j + 1]), __float_as_uint(v[j + 2]),
+                                       __float_as_uint(v[j + 3]));
+            if (q == rank)
+              *reinterpret_cast<uint4*>(dst + c0 + j) = u;
+            else if (*abort == 0)
+              st_async_v4(cluster_addr(dst + c0 + j, q), u, cluster_addr(bbar, q));
+          }
         }
       }
       tc_fence_before();
       __syncthreads();
       if (tid == 0)  // slots 2, 3 free: next layer's QKV
         for (int i = 2; i < 4; ++i) issue(q0 + kLayerChunks + i);
-      cluster.sync();  // every rank's partials of this rank's rows arrived
-      // h = silu(gate) * up for this rank's 16 SwiGLU columns, partials summed in rank order
-      for (int i = tid; i < kTokTile * 16; i += kThr) {
-        const int t = i >> 4;
-        const int cc = i & 15;
-        float g = 0.f, u = 0.f;
-#pragma unroll
-        for (int src = 0; src < kCl; ++src) {
-          g += recv[(src * 32 + cc) * kTokTile + t];
-          u += recv[(src * 32 + 16 + cc) * kTokTile + t];
-        }
-        *reinterpret_cast<__half*>(hsl + sw128_offset(kTokTile, t, rank * 16 + cc)) =
-            __float2half_rn(__fdividef(g, 1.f + __expf(-g)) * u);
-      }
+      xwait(bbar, par);  // every partner's partial sums of x^2 and gate/up partials
+      if (tid == 0 && *abort == 0) arm(bbar, FSX_B_BYTES);
+      compute_rstd();
       __syncthreads();
-      // this rank's 16 columns (two 16-byte units per token row) to the partners
-      for (int i = tid; i < kTokTile * 2 * (kCl - 1); i += kThr) {
-        const int peer_i = i / (kTokTile * 2);
-        const int rest = i - peer_i * kTokTile * 2;
-        const int t = rest >> 1;
-        const int u = rank * 2 + (rest & 1);
-        const int peer = peer_i + (peer_i >= rank ? 1 : 0);
-        const uint32_t off = sw128_offset(kTokTile, t, u * 8);
-        st_cluster_v4(cluster_addr(hsl + off, peer), *reinterpret_cast<const uint4*>(hsl + off));
+      // h = silu(gate) * up for this rank's 16 SwiGLU columns: K partials summed in rank
+      // order and scaled by 1 / rms; 8 columns a thread -> the swizzled slice here and in
+      // every partner
+      for (int i = tid; i < kTokTile * 2; i += kThr) {
+        const int t = i >> 1;
+        const int c8 = (i & 1) * 8;
+        const float r = rstd[t];
+        uint32_t hp[4];
+#pragma unroll
+        for (int j = 0; j < 8; j += 2) {
+          float hv[2];
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int cc = c8 + j + e;
+            float g = 0.f, u = 0.f;
+#pragma unroll
+            for (int src = 0; src < kCl; ++src) {
+              g += recv[(src * 32 + cc) * kTokTile + t];
+              u += recv[(src * 32 + 16 + cc) * kTokTile + t];
+            }
+            g *= r;
+            u *= r;
+            hv[e] = __fdividef(g, 1.f + __expf(-g)) * u;
+          }
+          hp[j >> 1] = pack_half2(hv[0], hv[1]);
+        }
+        const uint4 hv4 = make_uint4(hp[0], hp[1], hp[2], hp[3]);
+        unsigned char* dst = hsl + sw128_offset(kTokTile, t, rank * 16 + c8);
+        *reinterpret_cast<uint4*>(dst) = hv4;
+        if (t < T && *abort == 0) {
+#pragma unroll
+          for (int pi = 1; pi < kCl; ++pi) {
+            const int peer = (rank + pi) & (kCl - 1);
+            st_async_v4(cluster_addr(dst, peer), hv4, cluster_addr(hbar, peer));
+          }
+        }
       }
-      asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
-      cluster.sync();  // SwiGLU slice complete everywhere
-      // --- W_d: 128 output columns over the cluster's 64 SwiGLU inputs (slot 4)
-      if (warp == 0) {
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      xwait(hbar, par);  // the partners' SwiGLU columns
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the SwiGLU slice -> tensor core
+      __syncthreads();
+      if (tid == 0 && *abort == 0) arm(hbar, FSX_H_BYTES);
+      // --- W_d: 128 output columns over the cluster's 64 SwiGLU inputs (slot 4); warp w: K step w
+      if (warp < kNAcc) {
         tc_fence_after();
         const bool ok = wait_chunk(q0 + kPersistAChunks + 2);
-        if (ok && lane == 0) mma_slice(ring_a + 4 * kSlotBytes, smem_addr(hsl), true);
+        if (ok && lane == 0) mma_k(warp, ring_a + 4 * kSlotBytes, smem_addr(hsl), warp, 1, true);
         __syncwarp();
         if (lane == 0) umma_commit(mma_bar);
         __syncwarp();
       }
+      float4 resb[6];
+      if (c == 0) load_residual(Xm, rank * 128, resb);  // cluster 0 adds the residual itself
       wait_mma();
       tmem_to_dstT();
       if (tid == 0)  // slots 4, 5 free: next layer's QKV
         for (int i = 4; i < kSlots; ++i) issue(q0 + kLayerChunks + i);
       float* Xn = X0 + static_cast<size_t>((sA + 2) % 3) * xs;
-      scatter_add(Xn, Xm, rank * 128, c == 0);
+      scatter_add(Xn, rank * 128, resb, c == 0);
       arrive(p.counters + sA + 2);
     }
   }
@@ -1012,6 +1079,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
               : "r"(smem_addr(full + q % kSlots)), "r"(static_cast<uint32_t>((q / kSlots) & 1))
               : "memory");
       }
+  // no CTA leaves while a partner may still write into its shared memory
+  cluster.sync();
   tc_fence_before();
   __syncthreads();
   if (warp == 0)
@@ -1029,10 +1098,10 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         ss += v * v;
       }
       ss = warp_sum(ss);
-      const float rstd = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
+      const float rstd_j = rsqrtf(ss / static_cast<float>(d) + 1e-6f);
       float o0 = 0.f, o1 = 0.f;
       for (int c = lane; c < d; c += 32) {
-        const float n = __ldcg(xr + c) * rstd * p.final_norm[c];
+        const float n = __ldcg(xr + c) * rstd_j * p.final_norm[c];
         o0 += p.head_w[c] * n;
         o1 += p.head_w[d + c] * n;
       }
@@ -1045,6 +1114,13 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     }
   }
 }
+#undef FSX_T
+#undef FSX_X_BYTES
+#undef FSX_RS_BYTES
+#undef FSX_AG_BYTES
+#undef FSX_B_BYTES
+#undef FSX_H_BYTES
+#undef FSX_Q_BYTES
 
 }  // namespace
 
