@@ -134,34 +134,42 @@ __device__ __forceinline__ uint32_t cluster_addr(const void* local, int rank) {
 // bytes the partners will deliver by st.async.
 __device__ __forceinline__ void arm(uint64_t* bar, uint32_t bytes) { mbar_arrive_expect_tx(bar, bytes); }
 
-// tensor memory -> registers: 16 consecutive fp32 columns of each of the four
-// accumulators, added in accumulator order (two loads in flight at a time)
-__device__ __forceinline__ void tmem_ld16_x2(uint32_t taddr, uint32_t (&r)[2][16]) {
-#pragma unroll
-  for (int a = 0; a < 2; ++a)
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[a][0]), "=r"(r[a][1]), "=r"(r[a][2]), "=r"(r[a][3]), "=r"(r[a][4]), "=r"(r[a][5]), "=r"(r[a][6]),
-          "=r"(r[a][7]), "=r"(r[a][8]), "=r"(r[a][9]), "=r"(r[a][10]), "=r"(r[a][11]), "=r"(r[a][12]), "=r"(r[a][13]),
-          "=r"(r[a][14]), "=r"(r[a][15])
-        : "r"(taddr + static_cast<uint32_t>(a) * kAccCols));
-#pragma unroll
-  for (int a = 0; a < 2; ++a)
-    asm volatile("tcgen05.wait::ld.sync.aligned;"
-                 : "+r"(r[a][0]), "+r"(r[a][1]), "+r"(r[a][2]), "+r"(r[a][3]), "+r"(r[a][4]), "+r"(r[a][5]),
-                   "+r"(r[a][6]), "+r"(r[a][7]), "+r"(r[a][8]), "+r"(r[a][9]), "+r"(r[a][10]), "+r"(r[a][11]),
-                   "+r"(r[a][12]), "+r"(r[a][13]), "+r"(r[a][14]), "+r"(r[a][15])
-                 :
-                 : "memory");
+// tensor memory -> registers: N (16 or 32) consecutive fp32 columns of each of the four
+// accumulators, all loads in flight before one wait, added in accumulator order
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t (&r)[N]);
+template <>
+__device__ __forceinline__ void tmem_ld_cols<16>(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
 }
-__device__ __forceinline__ void tmem_ld16_sum4(uint32_t taddr, float (&v)[16]) {
-  uint32_t r[2][16];
-  tmem_ld16_x2(taddr, r);
+template <>
+__device__ __forceinline__ void tmem_ld_cols<32>(uint32_t taddr, uint32_t (&r)[32]) {
+  tmem_ld32_issue(taddr, r);
+}
+// the wait for every TMEM load of this thread; the registers are tied to it so that
+// no use of them is scheduled before it (the first wait completes all loads)
+__device__ __forceinline__ void tmem_wait_tied(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+               :
+               : "memory");
+}
+__device__ __forceinline__ void tmem_wait_tied(uint32_t (&r)[32]) { tmem_wait_ld32(r); }
+template <int N>
+__device__ __forceinline__ void tmem_ld_sum4(uint32_t taddr, float (&v)[N]) {
+  uint32_t r[kNAcc][N];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[0][i]) + __uint_as_float(r[1][i]);
-  tmem_ld16_x2(taddr + 2 * kAccCols, r);
+  for (int a = 0; a < kNAcc; ++a) tmem_ld_cols<N>(taddr + static_cast<uint32_t>(a) * kAccCols, r[a]);
 #pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = (v[i] + __uint_as_float(r[0][i])) + __uint_as_float(r[1][i]);
+  for (int a = 0; a < kNAcc; ++a) tmem_wait_tied(r[a]);
+#pragma unroll
+  for (int i = 0; i < N; ++i)
+    v[i] = ((__uint_as_float(r[0][i]) + __uint_as_float(r[1][i])) + __uint_as_float(r[2][i])) + __uint_as_float(r[3][i]);
 }
 
 // Bounded wait until *counter >= target (one thread polls, the CTA follows).
@@ -366,18 +374,24 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   // 8-column unit xu of rows xr0, xr0 + 16, xr0 + 32.
   const int xu = tid & 15;
   const int xr0 = tid >> 4;
-  // fp32 columns of this thread's rows -> fp16 x image (local, and the partners when
-  // `send_x`), per-token partial sums of x^2 -> gss[rank] here and in the partners;
-  // the partners' `peer_bar` counts the bytes
-  auto load_quarter = [&](const float* Xs, int col0, int k0, bool send_x, uint64_t* peer_bar) {
+  // this thread's fp32 columns of x (issued first thing after a phase's wait)
+  auto load_x = [&](const float* Xs, int col0, float4 (&xv)[3][2]) {
 #pragma unroll
     for (int i = 0; i < 3; ++i) {
       const int r = xr0 + 16 * i;
-      float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
-      if (r < T) {
-        a = ld_cg4(Xs + static_cast<size_t>(r) * d + col0 + xu * 8);
-        b = ld_cg4(Xs + static_cast<size_t>(r) * d + col0 + xu * 8 + 4);
-      }
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+        xv[i][h] = r < T ? ld_cg4(Xs + static_cast<size_t>(r) * d + col0 + xu * 8 + 4 * h) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  };
+  // those columns -> fp16 x image (local, and the partners when `send_x`), per-token
+  // partial sums of x^2 -> gss[rank] here and in the partners; the partners'
+  // `peer_bar` counts the bytes
+  auto convert_send = [&](const float4 (&xv)[3][2], int k0, bool send_x, uint64_t* peer_bar) {
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+      const int r = xr0 + 16 * i;
+      const float4 a = xv[i][0], b = xv[i][1];
       float ss = a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w + b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
 #pragma unroll
       for (int o = 8; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);  // the row's 16 threads
@@ -434,12 +448,16 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   auto tmem_to_dstT = [&]() {
     const int col = (warp & 3) * 32 + lane;
     const uint32_t taddr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
-    for (int c0 = warp < 4 ? 0 : 32; c0 < (warp < 4 ? 32 : 48); c0 += 16) {
-      float v[16];
-      __syncwarp();
-      tmem_ld16_sum4(taddr + static_cast<uint32_t>(c0), v);
+    if (warp < 4) {
+      float v[32];
+      tmem_ld_sum4<32>(taddr, v);
 #pragma unroll
-      for (int j = 0; j < 16; ++j) dstT[(c0 + j) * kDS + col] = v[j];
+      for (int j = 0; j < 32; ++j) dstT[j * kDS + col] = v[j];
+    } else {
+      float v[16];
+      tmem_ld_sum4<16>(taddr + 32u, v);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) dstT[(32 + j) * kDS + col] = v[j];
     }
     tc_fence_before();
     __syncthreads();
@@ -584,6 +602,12 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   }
   arrive(p.counters + 0);
 
+  // this CTA's share of the residual buffer each phase zeroes
+  const int zA0 = static_cast<int>(static_cast<long long>(n_elem) * cta / G);
+  const int zA1 = static_cast<int>(static_cast<long long>(n_elem) * (cta + 1) / G);
+  const int zB0 = static_cast<int>(static_cast<long long>(n_elem) * cta / n_b_ctas);
+  const int zB1 = static_cast<int>(static_cast<long long>(n_elem) * (cta + 1) / n_b_ctas);
+
   int q0 = 0;  // first ring position of the current layer
   const float scale_log2 = 1.4426950408889634f * rsqrtf(static_cast<float>(kD));
 
@@ -599,15 +623,15 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
 
     // =========================== phase A ===========================
     wait_counter(p.counters + sA, sA == 0 ? G : n_b_ctas, p.status, abort);
-    // zero the buffer phase B accumulates into
     {
-      const int e0 = static_cast<int>(static_cast<long long>(n_elem) * cta / G);
-      const int e1 = static_cast<int>(static_cast<long long>(n_elem) * (cta + 1) / G);
-      for (int e = e0 + tid; e < e1; e += kThr) __stcg(Xz + e, 0.f);
+      float4 xv[3][2];
+      load_x(Xc, rank * 128, xv);
+      // zero the buffer phase B accumulates into (while the loads are in flight)
+      for (int e = zA0 + tid; e < zA1; e += kThr) __stcg(Xz + e, 0.f);
+      // this rank's 128 columns of x -> fp16 image here and in the partners (K slices
+      // 2 rank, 2 rank + 1), partial sums of x^2 to every rank
+      convert_send(xv, rank * 128, true, xbar + rank);
     }
-    // this rank's 128 columns of x -> fp16 image here and in the partners (K slices
-    // 2 rank, 2 rank + 1), partial sums of x^2 to every rank
-    load_quarter(Xc, rank * 128, rank * 128, true, xbar + rank);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the local quarter -> tensor core
     __syncthreads();
 
@@ -649,12 +673,16 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       const uint32_t taddr = tmem + (static_cast<uint32_t>(kind * 32) << 16);
       const int c_lo = warp < 4 ? 0 : 32;
       const int c_hi = warp < 4 ? 32 : 48;
-      for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
-        float v[16];
-        __syncwarp();
-        tmem_ld16_sum4(taddr + static_cast<uint32_t>(c0), v);
+      if (warp < 4) {
+        float v[32];
+        tmem_ld_sum4<32>(taddr, v);
 #pragma unroll
-        for (int j = 0; j < 16; ++j) b[(c0 + j) * kQS + dim] = __float2half_rn(v[j] * rstd[c0 + j]);
+        for (int j = 0; j < 32; ++j) b[j * kQS + dim] = __float2half_rn(v[j] * rstd[j]);
+      } else {
+        float v[16];
+        tmem_ld_sum4<16>(taddr + 32u, v);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) b[(32 + j) * kQS + dim] = __float2half_rn(v[j] * rstd[32 + j]);
       }
       __syncwarp();
       // this warp's token rows below T (dims 32 rank .. + 31, four 16-byte units a row): q to
@@ -844,11 +872,13 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     // --- merge the 4 splits: every row's normalised fp32 partial and log-sum-exp go
     // straight from the registers to the rank that owns the row (st.async to the partners)
     if (warp < 6 && *abort == 0) {
-      auto put2 = [&](float* ptr, int dst, float a, float b) {
+      auto put4 = [&](float* ptr, int dst, float a, float b, float c, float e) {
         if (dst == rank)
-          *reinterpret_cast<float2*>(ptr) = make_float2(a, b);
+          *reinterpret_cast<float4*>(ptr) = make_float4(a, b, c, e);
         else
-          st_async_v2(cluster_addr(ptr, dst), __float_as_uint(a), __float_as_uint(b), cluster_addr(rsbar, dst));
+          st_async_v4(cluster_addr(ptr, dst),
+                      make_uint4(__float_as_uint(a), __float_as_uint(b), __float_as_uint(c), __float_as_uint(e)),
+                      cluster_addr(rsbar, dst));
       };
       auto put1 = [&](float* ptr, int dst, float a) {
         if (dst == rank)
@@ -864,11 +894,20 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       const float inv1 = l_run[1] > 0.f ? 1.f / l_run[1] : 0.f;
       float* d0 = recv + (rank * kRowsPerRank + qr0 - own0 * kRowsPerRank) * kD;
       float* d1 = recv + (rank * kRowsPerRank + qr1 - own1 * kRowsPerRank) * kD;
+      // lanes 2j and 2j + 1 hold columns 4j'..4j'+3 of rows qr0 and qr1 in pairs: the even
+      // lane sends row qr0's four, the odd lane row qr1's (one 16-byte store each)
+      const bool odd = (lane & 1) != 0;
 #pragma unroll
       for (int nb = 0; nb < 8; ++nb) {
         const int c = kh * 64 + nb * 8 + 2 * (lane & 3);
-        put2(d0 + c, own0, o_fin[nb][0] * inv0, o_fin[nb][1] * inv0);
-        put2(d1 + c, own1, o_fin[nb][2] * inv1, o_fin[nb][3] * inv1);
+        const float a0 = o_fin[nb][0] * inv0, a1 = o_fin[nb][1] * inv0;
+        const float b0 = o_fin[nb][2] * inv1, b1 = o_fin[nb][3] * inv1;
+        const float g0 = __shfl_xor_sync(0xffffffffu, odd ? a0 : b0, 1);
+        const float g1 = __shfl_xor_sync(0xffffffffu, odd ? a1 : b1, 1);
+        if (!odd)
+          put4(d0 + c, own0, a0, a1, g0, g1);
+        else
+          put4(d1 + c - 2, own1, g0, g1, b0, b1);
       }
       if (kh == 0 && (lane & 3) == 0) {
         put1(recv_lse + rank * kRowsPerRank + qr0 - own0 * kRowsPerRank, own0,
@@ -951,14 +990,15 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     if (in_b) {
       const int c = head;  // SwiGLU column block 64c..64c+63
       wait_counter(p.counters + sA + 1, G, p.status, abort);
-      {  // zero the buffer the next phase A accumulates into (this layer's input is consumed)
-        const int e0 = static_cast<int>(static_cast<long long>(n_elem) * cta / n_b_ctas);
-        const int e1 = static_cast<int>(static_cast<long long>(n_elem) * (cta + 1) / n_b_ctas);
-        for (int e = e0 + tid; e < e1; e += kThr) __stcg(Xc + e, 0.f);
+      {
+        float4 xv[3][2];
+        load_x(Xm, rank * 128, xv);
+        // zero the buffer the next phase A accumulates into (this layer's input is consumed)
+        for (int e = zB0 + tid; e < zB1; e += kThr) __stcg(Xc + e, 0.f);
+        // this rank's 128 columns of x -> fp16 K slices 0, 1 here (no exchange: each CTA runs
+        // the gate/up MMAs over its own K quarter), partial sums of x^2 to every rank
+        convert_send(xv, 0, false, bbar);
       }
-      // this rank's 128 columns of x -> fp16 K slices 0, 1 here (no exchange: each CTA runs
-      // the gate/up MMAs over its own K quarter), partial sums of x^2 to every rank
-      load_quarter(Xm, rank * 128, 0, false, bbar);
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // visible to the tensor core
       __syncthreads();
       // gate/up over this rank's K quarter: D[128 rows x 48 tokens], rows 32s..32s+31 = the
@@ -980,12 +1020,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         const int q = warp & 3;
         const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16);
         float* dst = recv + (rank * 32 + lane) * kTokTile;
-        for (int c0 = warp < 4 ? 0 : 32; c0 < (warp < 4 ? 32 : 48); c0 += 16) {
-          float v[16];
-          __syncwarp();
-          tmem_ld16_sum4(taddr + static_cast<uint32_t>(c0), v);
-#pragma unroll
-          for (int j = 0; j < 16; j += 4) {
+        auto put = [&](const float* v, int c0, int n) {
+          for (int j = 0; j < n; j += 4) {
             const uint4 u = make_uint4(__float_as_uint(v[j]), __float_as_uint(v[j + 1]), __float_as_uint(v[j + 2]),
                                        __float_as_uint(v[j + 3]));
             if (q == rank)
@@ -993,6 +1029,15 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
             else if (*abort == 0)
               st_async_v4(cluster_addr(dst + c0 + j, q), u, cluster_addr(bbar, q));
           }
+        };
+        if (warp < 4) {
+          float v[32];
+          tmem_ld_sum4<32>(taddr, v);
+          put(v, 0, 32);
+        } else {
+          float v[16];
+          tmem_ld_sum4<16>(taddr + 32u, v);
+          put(v, 32, 16);
         }
       }
       tc_fence_before();
