@@ -19,7 +19,12 @@
 //     at the start of every call, the partial slots are fully rewritten;
 //   * the first call on each device looks the array's device address up
 //     (cudaGetSymbolAddress) with that device current; make that first call
-//     before capturing any stream.
+//     before capturing any stream. The address is kept for the life of the
+//     process, so it does not survive a reset of the device's context
+//     (cudaDeviceReset): do not use these entry points after one;
+//   * device-side argument errors (offsets that decrease or are negative) and
+//     timeouts are recorded in the array's status word, not in a caller buffer:
+//     fsx_attention_noalloc_status reads and clears it.
 #include <cuda_runtime.h>
 
 #include <cstdio>
@@ -46,6 +51,22 @@ void* g_scratch_ptr[kMaxDevices] = {};
 fsx_status noalloc_fail(fsx_status s, const char* msg) {
   fsx::set_error_message(msg);
   return s;
+}
+
+// Device address of the static scratch on the current device (looked up once per device).
+fsx_status scratch_base(void** base) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+    return noalloc_fail(FSX_ERR_CUDA, "cudaGetDevice failed or device index out of range");
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (g_scratch_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || p == nullptr) return noalloc_fail(FSX_ERR_CUDA, cudaGetErrorString(e));
+    g_scratch_ptr[dev] = p;
+  }
+  *base = g_scratch_ptr[dev];
+  return FSX_OK;
 }
 
 }  // namespace
@@ -77,27 +98,16 @@ extern "C" fsx_status fsx_attention_noalloc(const void* d_q, long long q_stride,
     return noalloc_fail(FSX_ERR_INVALID_ARG, msg);
   }
 
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
-    return noalloc_fail(FSX_ERR_CUDA, "cudaGetDevice failed or device index out of range");
   void* base = nullptr;
-  {
-    std::lock_guard<std::mutex> lock(g_scratch_mu);
-    if (g_scratch_ptr[dev] == nullptr) {
-      void* p = nullptr;
-      const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-      if (e != cudaSuccess || p == nullptr) return noalloc_fail(FSX_ERR_CUDA, cudaGetErrorString(e));
-      g_scratch_ptr[dev] = p;
-    }
-    base = g_scratch_ptr[dev];
-  }
+  const fsx_status bs = scratch_base(&base);
+  if (bs != FSX_OK) return bs;
   if (fsx::attention_set_attributes() != cudaSuccess)
     return noalloc_fail(FSX_ERR_CUDA, "cudaFuncSetAttribute failed");
 
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int* status = static_cast<int*>(base);
   float* part = reinterpret_cast<float*>(static_cast<unsigned char*>(base) + kStatusSlot);
-  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), st);
+  cudaError_t e = cudaMemsetAsync(status, 0, 2 * sizeof(int), st);  // error word, range word
   if (e != cudaSuccess) return noalloc_fail(FSX_ERR_CUDA, cudaGetErrorString(e));
 
   fsx::AttnArgs a{};
@@ -124,5 +134,25 @@ extern "C" fsx_status fsx_attention_noalloc(const void* d_q, long long q_stride,
   a.status = status;
   e = fsx::launch_attention(a, B, cache_dtype, st, false);
   if (e != cudaSuccess) return noalloc_fail(FSX_ERR_CUDA, cudaGetErrorString(e));
+  return FSX_OK;
+}
+
+// The device status word of the static scratch: synchronises `stream` (the stream of
+// the calls to check), returns the word and clears it. Copies one int each way; no
+// allocation.
+extern "C" fsx_status fsx_attention_noalloc_status(void* stream) {
+  fsx::set_error_message("");
+  void* base = nullptr;
+  const fsx_status bs = scratch_base(&base);
+  if (bs != FSX_OK) return bs;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int word[2] = {0, 0};  // error word, range word
+  cudaError_t e = cudaMemcpyAsync(word, base, 2 * sizeof(int), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(base, 0, 2 * sizeof(int), st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return noalloc_fail(FSX_ERR_CUDA, cudaGetErrorString(e));
+  if (word[0] == static_cast<int>(FSX_ERR_TIMEOUT)) return noalloc_fail(FSX_ERR_TIMEOUT, "a device-side wait timed out");
+  if (word[0] != 0) return noalloc_fail(FSX_ERR_DEVICE_ARG, "device-side check: cache offsets negative or decreasing");
+  if (word[1] != 0) return noalloc_fail(FSX_ERR_RANGE, "cache values beyond the fp16 range were saturated to +-65504");
   return FSX_OK;
 }

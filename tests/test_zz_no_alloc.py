@@ -2,7 +2,9 @@
 allocate device memory while running (it keeps its scratch in a static array
 inside the library). Its results must equal those of fsx_attention, which
 uses a caller scratch buffer, on two calls in a row with different inputs
-(the second call must not see the first call's leftovers)."""
+(the second call must not see the first call's leftovers). Device-side
+argument errors land in the static array's status word, which
+fsx_attention_noalloc_status reads and clears."""
 from __future__ import annotations
 
 import numpy as np
@@ -79,3 +81,29 @@ def test_no_alloc_rejects_requests_beyond_its_scratch():
                               "bf16", c["off"], c["B"], H, too_many, out, None)
     assert e.value.status == fsx.FSX_ERR_INVALID_ARG
     assert "scratch" in str(e.value)
+
+
+def test_no_alloc_reports_device_side_offset_errors_through_its_status_word():
+    c = _inputs([50, 30], seed=5)
+    H = c["H"]
+    assert fsx.attention_noalloc_status() == fsx.FSX_OK  # nothing pending from earlier calls
+    # offsets [0, 50, 20]: vehicle 1's range runs backwards; its rows must stay untouched
+    bad = torch.as_tensor(np.array([0, 50, 20], dtype=np.int64), device="cuda")
+    out = torch.full((c["B"] * c["n_q"], H * D), float("nan"), device="cuda", dtype=torch.float16)
+    fsx.attention_noalloc(c["q"], H * D, c["ko"], c["vo"], H * D, c["n_q"], c["n_own"], c["kc"], c["vc"], "bf16",
+                          bad, c["B"], H, 1, out, None)
+    assert fsx.attention_noalloc_status() == fsx.FSX_ERR_DEVICE_ARG
+    assert torch.isnan(out[c["n_q"]:].float()).all()
+    assert fsx.attention_noalloc_status() == fsx.FSX_OK  # read-and-clear
+    # a negative first offset with one vehicle: nothing is written at all
+    neg = torch.as_tensor(np.array([-4, 20], dtype=np.int64), device="cuda")
+    out1 = torch.full((c["n_q"], H * D), float("nan"), device="cuda", dtype=torch.float16)
+    fsx.attention_noalloc(c["q"], H * D, c["ko"], c["vo"], H * D, c["n_q"], c["n_own"], c["kc"], c["vc"], "bf16",
+                          neg, 1, H, 1, out1, None)
+    assert fsx.attention_noalloc_status() == fsx.FSX_ERR_DEVICE_ARG
+    assert torch.isnan(out1.float()).all()
+    # the next good call runs normally and leaves the word clear
+    ref_out, _ = _with_buffer(c, 5)
+    out2, _ = _no_alloc(c, 5)
+    assert fsx.attention_noalloc_status() == fsx.FSX_OK
+    assert _row_err(out2, ref_out).max() < 2e-3
