@@ -23,8 +23,14 @@
  *   - Precision: weights are stored as fp16 (round-to-nearest-even from the
  *     fp32 host copy; exact for bf16-valued weights), GEMM and attention
  *     operands are fp16 with fp32 accumulation, the residual stream, RMSNorm,
- *     softmax statistics and the head are fp32. Cache values are converted to
- *     fp16 on load and must lie within +-65504.
+ *     softmax statistics and the head are fp32. Cache values the kernels
+ *     convert to fp16 (every key; the values too, except in the bf16 tensor-core
+ *     attention of batched ticks) are expected within +-65504. A value beyond
+ *     that (a bf16 magnitude of 65536 or more, an fp32 magnitude that rounds
+ *     past 65504, infinity or NaN) is saturated to +-65504 instead of becoming
+ *     an infinity that would turn the softmax into NaN, and the status read by
+ *     fsx_get_status becomes FSX_ERR_RANGE: the results of that tick are those of
+ *     the saturated cache, not of the caller's values.
  */
 #ifndef FSX_H
 #define FSX_H
@@ -45,8 +51,11 @@ typedef enum {
   FSX_ERR_OOM = 3,          /* a device or host allocation failed              */
   FSX_ERR_CUDA = 4,         /* a CUDA runtime call failed (see fsx_last_error) */
   FSX_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up              */
-  FSX_ERR_DEVICE_ARG = 6    /* device-side check: offsets not non-decreasing,
+  FSX_ERR_DEVICE_ARG = 6,   /* device-side check: offsets not non-decreasing,
                                negative, or beyond max_total_cache_tokens      */
+  FSX_ERR_RANGE = 7         /* device-side check: a cache value lay outside the
+                               fp16 range (see Precision); it was saturated to
+                               +-65504 and the tick completed on that value    */
 } fsx_status;
 
 typedef enum { FSX_F32 = 0, FSX_BF16 = 1 } fsx_dtype;
@@ -147,8 +156,13 @@ fsx_status fsx_tick_ranges_debug(fsx_handle h, const void* const* k_cache, const
                                  const int64_t* d_starts, const int64_t* d_offsets, int B, const void* d_frames,
                                  float* d_waypoints, void* d_attn_out, void* stream);
 
-/* Synchronises `stream`, then returns and clears the device status word
- * (FSX_OK, FSX_ERR_DEVICE_ARG or FSX_ERR_TIMEOUT). */
+/* Status of the handle's ticks since the previous call. Not a passage of the
+ * paper: the error path of the tick (Sec. 3.3 runs it every 50 ms, so a failed
+ * tick must be detectable without stopping the stream). Synchronises `stream`
+ * (the stream of the ticks to check), then returns and clears the device status
+ * block: FSX_OK, FSX_ERR_DEVICE_ARG, FSX_ERR_TIMEOUT (errors: that tick's
+ * kernels skipped their work) or FSX_ERR_RANGE (the tick completed on saturated
+ * cache values). Errors take precedence over FSX_ERR_RANGE. */
 fsx_status fsx_get_status(fsx_handle h, void* stream);
 
 /* Thread-local message describing the last failure on this thread ("" if none). */
@@ -216,6 +230,12 @@ fsx_status fsx_attention(const void* d_q, long long q_stride,
  * that array, so calls whose kernels overlap on the GPU race and must be
  * serialised by the caller. The first call on each device resolves the array's
  * device address with that device current; make it before capturing a stream.
+ * The resolved address is kept for the process: it does not survive a reset of
+ * the device's context (cudaDeviceReset), after which these entry points must
+ * not be used. Unlike fsx_attention, whose status word sits in the caller's
+ * workspace, device-side argument errors (cache offsets that are negative or
+ * decrease: the vehicle concerned writes no output row) are recorded in the
+ * static array; read them with fsx_attention_noalloc_status.
  * Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
 fsx_status fsx_attention_noalloc(const void* d_q, long long q_stride,
                                  const void* d_k_own, const void* d_v_own, long long own_stride,
@@ -223,6 +243,16 @@ fsx_status fsx_attention_noalloc(const void* d_q, long long q_stride,
                                  const void* d_k_cache, const void* d_v_cache, int cache_dtype,
                                  const int64_t* d_offsets, int B, int n_heads, int head_dim,
                                  int n_splits, void* d_out, float* d_lse, void* stream);
+
+/* The device status word of fsx_attention_noalloc's static array on the current
+ * device (the paper has no counterpart; it completes that entry point for the
+ * same callers). Synchronises `stream` -- the stream of the calls to check --
+ * then returns the word and clears it: FSX_OK, FSX_ERR_DEVICE_ARG (a call saw
+ * negative or decreasing cache offsets), FSX_ERR_TIMEOUT or FSX_ERR_RANGE (cache
+ * values saturated to the fp16 range, as in fsx_get_status). Copies two ints to
+ * the host and clears them on the device; allocates nothing. Calls still running
+ * on other streams may set the word afterwards. */
+fsx_status fsx_attention_noalloc_status(void* stream);
 
 /* ================================================================== cache append
  * The slow system's incremental forward (Sec. 1, Sec. 3.3): every K = 4 ticks

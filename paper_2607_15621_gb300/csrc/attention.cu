@@ -87,28 +87,31 @@ __device__ __forceinline__ void cp_async_wait_n(int n) {
 }
 
 template <typename CT>
-__device__ __forceinline__ void convert_unit(const unsigned char* raw, uint4* dst, bool own);
+__device__ __forceinline__ void convert_unit(const unsigned char* raw, uint4* dst, bool own, uint32_t& range);
 
-// bf16 cache rows: 16 raw bytes = 8 values -> 8 fp16
+// bf16 cache rows: 16 raw bytes = 8 values -> 8 fp16 (saturated, out-of-range values recorded)
 template <>
-__device__ __forceinline__ void convert_unit<__nv_bfloat16>(const unsigned char* raw, uint4* dst, bool own) {
+__device__ __forceinline__ void convert_unit<__nv_bfloat16>(const unsigned char* raw, uint4* dst, bool own,
+                                                            uint32_t& range) {
   const uint4 v = *reinterpret_cast<const uint4*>(raw);
   if (own) {
     *dst = v;
   } else {
-    *dst = make_uint4(bf16x2_to_half2(v.x), bf16x2_to_half2(v.y), bf16x2_to_half2(v.z), bf16x2_to_half2(v.w));
+    *dst = make_uint4(bf16x2_to_half2_sat(v.x, range), bf16x2_to_half2_sat(v.y, range),
+                      bf16x2_to_half2_sat(v.z, range), bf16x2_to_half2_sat(v.w, range));
   }
 }
 
 // fp32 cache rows: 32 raw bytes = 8 values -> 8 fp16 (own rows are fp16 in the first half)
 template <>
-__device__ __forceinline__ void convert_unit<float>(const unsigned char* raw, uint4* dst, bool own) {
+__device__ __forceinline__ void convert_unit<float>(const unsigned char* raw, uint4* dst, bool own, uint32_t& range) {
   if (own) {
     *dst = *reinterpret_cast<const uint4*>(raw);
   } else {
     const float4 a = *reinterpret_cast<const float4*>(raw);
     const float4 b = *reinterpret_cast<const float4*>(raw + 16);
-    *dst = make_uint4(pack_half2(a.x, a.y), pack_half2(a.z, a.w), pack_half2(b.x, b.y), pack_half2(b.z, b.w));
+    *dst = make_uint4(f32x2_to_half2_sat(a.x, a.y, range), f32x2_to_half2_sat(a.z, a.w, range),
+                      f32x2_to_half2_sat(b.x, b.y, range), f32x2_to_half2_sat(b.z, b.w, range));
   }
 }
 
@@ -264,6 +267,7 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
 
   const int n_chunks = empty_range ? 0 : static_cast<int>((kend - kbeg + kChunk - 1) / kChunk);
   for (int i = 0; i < kRawStages && i < n_chunks; ++i) issue_chunk(i, i);
+  uint32_t range = 0;  // a cache value outside the fp16 range was saturated
 
   for (int c = 0; c < n_chunks; ++c) {
     const int s = c % kRawStages;
@@ -288,8 +292,8 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
             uint4* kd = kt + swz(r, u);
             uint4* vd = vt + swz(r, u);
             if (r < rows) {
-              convert_unit<CT>(kr + static_cast<size_t>(r) * RB + u * SRC_UNIT, kd, false);
-              convert_unit<CT>(vr + static_cast<size_t>(r) * RB + u * SRC_UNIT, vd, false);
+              convert_unit<CT>(kr + static_cast<size_t>(r) * RB + u * SRC_UNIT, kd, false, range);
+              convert_unit<CT>(vr + static_cast<size_t>(r) * RB + u * SRC_UNIT, vd, false, range);
             } else {
               *kd = make_uint4(0u, 0u, 0u, 0u);
               *vd = make_uint4(0u, 0u, 0u, 0u);
@@ -304,8 +308,8 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
         if (r < rows) {
           const bool own = (c0 + r) >= L;
           const int off = own ? u * 16 : u * SRC_UNIT;
-          convert_unit<CT>(kr + static_cast<size_t>(r) * RB + off, kd, own);
-          convert_unit<CT>(vr + static_cast<size_t>(r) * RB + off, vd, own);
+          convert_unit<CT>(kr + static_cast<size_t>(r) * RB + off, kd, own, range);
+          convert_unit<CT>(vr + static_cast<size_t>(r) * RB + off, vd, own, range);
         } else {
           *kd = make_uint4(0u, 0u, 0u, 0u);
           *vd = make_uint4(0u, 0u, 0u, 0u);
@@ -420,6 +424,7 @@ __global__ void __launch_bounds__(kThreads, FSX_ATTN_MIN_CTAS) attn_splitkv_kern
       }
     }
   }
+  flag_range(p.status, range);
 
   // ---- write out
   const float inv0 = l_run[0] > 0.f ? 1.f / l_run[0] : 0.f;

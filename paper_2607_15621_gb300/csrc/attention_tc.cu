@@ -390,6 +390,7 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
     uint64_t* full = is_v ? vfull : kfull;
     uint64_t* empty = is_v ? vempty : kempty;
     bool ok = true;
+    uint32_t range = 0;  // a cache key outside the fp16 range was saturated
     for (int i = 0; ok && i < n_chunks; ++i) {
       if (i + 1 < n_chunks) cp_async_wait<1>();
       else cp_async_wait<0>();
@@ -405,7 +406,8 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
         for (int m = 0; m < kSlotKeys / 4; ++m) {
           uint4* ptr = reinterpret_cast<uint4*>(slot + tile128_off(pr0 + 4 * m, pu));
           const uint4 v = *ptr;
-          *ptr = make_uint4(bf16x2_to_half2(v.x), bf16x2_to_half2(v.y), bf16x2_to_half2(v.z), bf16x2_to_half2(v.w));
+          *ptr = make_uint4(bf16x2_to_half2_sat(v.x, range), bf16x2_to_half2_sat(v.y, range),
+                            bf16x2_to_half2_sat(v.z, range), bf16x2_to_half2_sat(v.w, range));
         }
       }
       fence_proxy_async();
@@ -416,6 +418,7 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
       }
     }
     cp_async_wait<0>();
+    flag_range(p.status, range);
   } else {
     // ---------------------------------------------------------------- softmax rows
     // Warp w owns query rows 16 w .. 16 w + 15 (tensor-memory lanes 32 w .. + 15).

@@ -10,7 +10,7 @@
 namespace fsx {
 
 // Status codes written into the device status word (mirrors fsx_status).
-enum : int { kStatusOk = 0, kStatusTimeout = 5, kStatusDeviceArg = 6 };
+enum : int { kStatusOk = 0, kStatusTimeout = 5, kStatusDeviceArg = 6, kStatusRange = 7 };
 
 // ~1 s bound for every device-side wait (globaltimer counts nanoseconds).
 constexpr unsigned long long kWaitLimitNs = 1000000000ull;
@@ -175,6 +175,31 @@ __device__ __forceinline__ float warp_sum(float v) {
 __device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
   __half2 h = __floats2half2_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Cache values converted to fp16 saturate at +-65504 instead of overflowing to
+// infinity (cvt .satfinite), and every such value is recorded: `range` collects
+// whether an input lay outside the fp16 range (a bf16 magnitude of 65536 or more,
+// infinity or NaN; an fp32 magnitude that rounds beyond 65504), and
+// flag_range() raises the second word of the status block, which the kernels do
+// not treat as an error (the tick continues on the saturated values) and the
+// host reports as FSX_ERR_RANGE.
+__device__ __forceinline__ uint32_t bf16x2_to_half2_sat(uint32_t v, uint32_t& range) {
+  const float lo = __uint_as_float(v << 16);
+  const float hi = __uint_as_float(v & 0xffff0000u);
+  range |= static_cast<uint32_t>((v & 0x7fffu) >= 0x4780u) | static_cast<uint32_t>(((v >> 16) & 0x7fffu) >= 0x4780u);
+  uint32_t r;
+  asm("cvt.rn.satfinite.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+__device__ __forceinline__ uint32_t f32x2_to_half2_sat(float lo, float hi, uint32_t& range) {
+  range |= static_cast<uint32_t>(!(fabsf(lo) < 65520.f)) | static_cast<uint32_t>(!(fabsf(hi) < 65520.f));
+  uint32_t r;
+  asm("cvt.rn.satfinite.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+__device__ __forceinline__ void flag_range(int* status, uint32_t range) {
+  if (range) *reinterpret_cast<volatile int*>(status + 1) = kStatusRange;
 }
 
 // Two bf16 (low half first) -> two fp16, via fp32 (bf16 -> fp32 is exact).

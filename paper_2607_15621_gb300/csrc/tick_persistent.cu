@@ -523,6 +523,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     }
     cp_async_commit();
   };
+  uint32_t range_seen = 0;  // a cache value outside the fp16 range was saturated
   // all threads: wait for chunk j and convert it to fp16 in place
   auto stage_ready = [&](int j) {
     const int younger = min(n_chunks - 1 - j, kNB - 1);  // groups of later chunks still in flight
@@ -558,8 +559,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
           const int key = r >= kStageKeys ? r - kStageKeys : r;
           if (r0 + it < kCvtIters && r < 2 * kStageKeys && key < n)
             *reinterpret_cast<uint4*>(kb + r * kRowStride + (i & 15) * 16) =
-                make_uint4(bf16x2_to_half2(v[it].x), bf16x2_to_half2(v[it].y), bf16x2_to_half2(v[it].z),
-                           bf16x2_to_half2(v[it].w));
+                make_uint4(bf16x2_to_half2_sat(v[it].x, range_seen), bf16x2_to_half2_sat(v[it].y, range_seen),
+                           bf16x2_to_half2_sat(v[it].z, range_seen), bf16x2_to_half2_sat(v[it].w, range_seen));
         }
       }
     } else {
@@ -578,7 +579,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
         if (live) {
           const float4 a = *reinterpret_cast<const float4*>(row + u * 32);
           const float4 b = *reinterpret_cast<const float4*>(row + u * 32 + 16);
-          o = make_uint4(pack_half2(a.x, a.y), pack_half2(a.z, a.w), pack_half2(b.x, b.y), pack_half2(b.z, b.w));
+          o = make_uint4(f32x2_to_half2_sat(a.x, a.y, range_seen), f32x2_to_half2_sat(a.z, a.w, range_seen),
+                         f32x2_to_half2_sat(b.x, b.y, range_seen), f32x2_to_half2_sat(b.z, b.w, range_seen));
         }
         __syncthreads();
         if (live) *reinterpret_cast<uint4*>(row + u * 16) = o;
@@ -1124,6 +1126,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
               : "r"(smem_addr(full + q % kSlots)), "r"(static_cast<uint32_t>((q / kSlots) & 1))
               : "memory");
       }
+  flag_range(p.status, range_seen);
   // no CTA leaves while a partner may still write into its shared memory
   cluster.sync();
   tc_fence_before();

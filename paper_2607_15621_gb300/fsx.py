@@ -24,6 +24,7 @@ FSX_ERR_OOM = 3
 FSX_ERR_CUDA = 4
 FSX_ERR_TIMEOUT = 5
 FSX_ERR_DEVICE_ARG = 6
+FSX_ERR_RANGE = 7
 FSX_F32 = 0
 FSX_BF16 = 1
 
@@ -91,6 +92,7 @@ def _load():
                                 vp, i32, i32, i32, i32, vp, vp, vp, ctypes.c_size_t, vp]),
         "fsx_attention_noalloc": (i32, [vp, ctypes.c_longlong, vp, vp, ctypes.c_longlong, i32, i32, vp, vp,
                                         i32, vp, i32, i32, i32, i32, vp, vp, vp]),
+        "fsx_attention_noalloc_status": (i32, [vp]),
         "fsx_append_create": (i32, [ctypes.POINTER(AppendConfig), ctypes.POINTER(AppendWeights), i32,
                                     ctypes.POINTER(vp)]),
         "fsx_append": (i32, [vp, vpp, vpp, vp, vp, i32, vp, vp, vp]),
@@ -120,7 +122,7 @@ def declared_symbols() -> list[str]:
             "fsx_get_status", "fsx_last_error",
             "fsx_destroy", "fsx_weight_bytes", "fsx_tick_launches", "fsx_set_kernel_timing",
             "fsx_kernel_time", "fsx_attention_workspace_bytes", "fsx_attention", "fsx_attention_noalloc",
-            "fsx_append_create", "fsx_append", "fsx_append_get_status", "fsx_append_weight_bytes",
+            "fsx_attention_noalloc_status", "fsx_append_create", "fsx_append", "fsx_append_get_status", "fsx_append_weight_bytes",
             "fsx_append_destroy"]
 
 
@@ -269,6 +271,12 @@ def attention_noalloc(q, q_stride, k_own, v_own, own_stride, n_q, n_own, k_cache
                                       _ptr(k_cache), _ptr(v_cache), code, _ptr(offsets), B, n_heads, 128,
                                       n_splits, _ptr(out), _ptr(lse), _stream(stream)))
     return out
+
+
+def attention_noalloc_status(stream=None) -> int:
+    """fsx_attention_noalloc_status: synchronises the stream, returns and clears the
+    device status word of the static scratch (FSX_OK, FSX_ERR_DEVICE_ARG or FSX_ERR_TIMEOUT)."""
+    return int(lib().fsx_attention_noalloc_status(_stream(stream)))
 
 
 class Append:
