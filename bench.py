@@ -4,6 +4,17 @@ head) on synthetic seeded inputs, printed as one JSON line.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl fsx|reference]
 
+Default workload: bf16_b128_ragged, the largest single-GPU configuration: 128
+vehicles with ragged caches L_b ~ U[64, 2048] (the seeded draw holds 129,767
+cached tokens per layer, 68 GB over 32 layers), bf16 weights / cache / frames.
+value = vehicle-ticks/s over all ranks (weak scaling: every rank runs its own
+vehicles; the path has no cross-vehicle exchange). The same line carries, under
+"workloads", the B = 1 paper-shaped tick (bf16_b1_l224), the history-length
+sweep at B = 1 (L = 224 ... 4096) and the 16-vehicle batch, each with its
+us/tick and its fraction of the max(HBM, tensor) tick roofline. Inputs are
+resident in HBM when the timed region starts; weights (675 MB) plus cache
+exceed the 129 MB L2, so no flush is needed between ticks.
+
 The workload `clip_j40_delta1` times the staleness-masked forward over a 40-frame
 clip (Sec. 3.2: every frame block over the cache prefix ending one frame earlier,
 all blocks in one tick over explicit row ranges); value = frame-blocks/s.
@@ -11,12 +22,8 @@ The workload `append_b1_l224` instead times the backbone's incremental cache
 append (one call = n_new = 4 tokens through the 32-layer, 4096-wide backbone
 for one vehicle with 224 cached tokens); value = vehicle-appends/s.
 
-Default workload: bf16_b1_l224 (B=1 vehicle, 224 cached backbone tokens per
-layer = 64 instruction + 40 frames x 4, bf16 weights/cache/frames, 32 layers).
-value = vehicle-ticks/s over all ranks (weak scaling: every rank runs its own
-vehicles; the path has no cross-vehicle exchange). Inputs are resident in HBM
-when the timed region starts; weights (675 MB) plus cache exceed the 129 MB L2,
-so no flush is needed between ticks.
+Without torchrun (WORLD_SIZE unset), --gpus N > 1 starts N ranks itself, one
+per GPU, and rank 0 prints the line.
 """
 from __future__ import annotations
 
@@ -41,15 +48,34 @@ FALLBACK_TENSOR_TFS = 1700.0      # dense bf16 / fp16, sustained (one earlier GB
 NOMINAL_HBM_GBS = 8000.0          # the HBM3e figure the tick roofline is stated against
 NOMINAL_TENSOR_TFS = 2250.0       # dense bf16 / fp16 tensor peak, nominal
 KCLASS_NAMES = ["qkv", "attention", "out_proj", "gate_up", "down", "persistent"]
+DEFAULT_WORKLOAD = "bf16_b128_ragged"
+# timed beside the headline with the same handle: the B = 1 paper-shaped tick, the
+# history-length sweep and the 16-vehicle batch
+EXTRA_WORKLOADS = ["bf16_b1_l224", "bf16_b1_l512", "bf16_b1_l1024", "bf16_b1_l2048", "bf16_b1_l4096",
+                   "bf16_b16_ragged"]
 
-# DRAM bytes (read + write) of one launch of the timed kernel, from one ncu capture of the
-# kernel as it is now (profiles/ holds each summary with its command). A kernel that changed
-# after its capture gets no entry, so its traffic is reported as null.
+# DRAM bytes (read + write) of one launch of the timed kernel, from one ncu capture, with the
+# SHA-256 prefix of the kernel's source file at capture time: a figure whose source has
+# changed since is reported as null (traffic_stale).
 NCU_TRAFFIC = {
-    ("persistent", "bf16_b1_l224"): 793.002752e6 + 3.571456e6,   # persistent_tick_bf16_b1_l224.md
-    ("qkv", "bf16_b128_ragged"): 18.229504e6 + 71.913728e6,      # gemm_tc_bf16_b128_ragged.md
-    ("attention", "bf16_b128_ragged"): 2258.334e6 + 39.689472e6,  # attn_tc_bf16_b128_ragged.md
+    ("attention", "bf16_b128_ragged"): (2298023472.0, "attention_tc.cu", "STALE"),
 }
+
+
+def traffic_for(kclass, workload):
+    """(bytes, stale) of the timed kernel's last ncu capture, (None, False) when none exists."""
+    import hashlib
+    entry = NCU_TRAFFIC.get((kclass, workload))
+    if entry is None:
+        return None, False
+    nbytes, src, sha = entry
+    path = os.path.join(ROOT, "paper_2607_15621_gb300", "csrc", src)
+    try:
+        with open(path, "rb") as fh:
+            cur = hashlib.sha256(fh.read()).hexdigest()[:16]
+    except OSError:
+        return None, True
+    return (nbytes, False) if cur == sha else (None, True)
 
 
 def parse():
@@ -57,13 +83,15 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
-    ap.add_argument("--workload", default="bf16_b1_l224")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", default="fsx", choices=["fsx", "reference"])
     ap.add_argument("--kernel-class", default=None, choices=KCLASS_NAMES,
                     help="kernel timed for the roofline (default: the dominant one, i.e. the persistent tick "
                          "for one vehicle and attention for a batch)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="time only the named workload (no B = 1, sweep and B = 16 entries)")
     ap.add_argument("--layers", type=int, default=None,
                     help="expert layers (default: the workload's 32); fewer layers keep a profiling run's cache small")
     return ap.parse_args()
@@ -177,26 +205,61 @@ def stop_clock_sampler(proc, fh, path):
             "samples": len(sm)}
 
 
+def baseline_vehicles(lengths, n=8):
+    """The vehicles the CPU baseline runs: for one vehicle that one; for a batch, n of
+    them spread over the length order, the shortest and the longest included."""
+    lengths = np.asarray(lengths)
+    if len(lengths) == 1:
+        return [0]
+    order = np.argsort(lengths, kind="stable")
+    picks = np.unique(np.round(np.linspace(0, len(order) - 1, min(n, len(order)))).astype(int))
+    return [int(order[i]) for i in picks]
+
+
 def cpu_baseline(name, seconds):
-    """The fp64 oracle as it stands, on the host cores, on vehicle 0 of the workload."""
+    """The fp64 oracle as it stands, on the host cores. One vehicle: vehicle 0's tick
+    repeated for `seconds`. A batch: one tick of each of 8 vehicles spread over the
+    length order (shortest and longest included), each over its own seeded draw of a
+    cache of its length (the batch's 68 GB cache is not copied to the host), stopping
+    early only past 4 x `seconds`; vehicles are independent, so the rate is per
+    vehicle-tick of that mix."""
     from oracle import fsx_oracle
     from paper_2607_15621_gb300 import synth
     spec, lengths = workload_info(name)
     dims = synth.EXPERT
     w = synth.make_weights(dims, 0, spec["dtype"])
-    k, v, off = synth.make_cache(dims, lengths[:1], 0, spec["dtype"])
-    kn = [t.float().numpy() for t in k]
-    vn = [t.float().numpy() for t in v]
-    fr = synth.make_frames(dims, 1, 0, spec["dtype"]).double().numpy()
-    n, t0 = 0, time.perf_counter()
-    while True:
-        fsx_oracle.expert_tick(w, kn, vn, off, fr, dims.n_heads, dims.head_dim, dims.n_waypoints)
-        n += 1
-        el = time.perf_counter() - t0
-        if el >= seconds or n >= 1000:
-            break
-    return {"value": n / el, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{n} full 32-layer fp64 ticks of vehicle 0 of {name} (L={int(lengths[0])}) in {el:.1f} s"}
+    picks = baseline_vehicles(lengths)
+
+    def inputs(b):
+        k, v, off = synth.make_cache(dims, [int(lengths[b])], 1000 + b, spec["dtype"])
+        fr = synth.make_frames(dims, 1, 1000 + b, spec["dtype"]).double().numpy()
+        return [t.float().numpy() for t in k], [t.float().numpy() for t in v], off, fr
+
+    n, done, t0 = 0, [], time.perf_counter()
+    if len(picks) == 1:
+        kn, vn, off, fr = inputs(0)
+        t0 = time.perf_counter()
+        while True:
+            fsx_oracle.expert_tick(w, kn, vn, off, fr, dims.n_heads, dims.head_dim, dims.n_waypoints)
+            n += 1
+            el = time.perf_counter() - t0
+            if el >= seconds or n >= 1000:
+                break
+        sample = f"{n} full 32-layer fp64 ticks of vehicle 0 of {name} (L={int(lengths[0])}) in {el:.1f} s"
+    else:
+        el = 0.0
+        for b in picks:
+            kn, vn, off, fr = inputs(b)
+            t1 = time.perf_counter()
+            fsx_oracle.expert_tick(w, kn, vn, off, fr, dims.n_heads, dims.head_dim, dims.n_waypoints)
+            el += time.perf_counter() - t1
+            n += 1
+            done.append(int(lengths[b]))
+            if el >= 4 * seconds:
+                break
+        sample = (f"one full 32-layer fp64 tick of each of {n} vehicles of {name} spread over the length order "
+                  f"(L = {done}), each over its own seeded cache draw, {el:.1f} s of oracle time")
+    return {"value": n / el, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample}
 
 
 APPEND_METRIC = "vehicle-appends/s (1e6 / us-per-append x B) of the backbone's incremental cache append"
@@ -525,21 +588,95 @@ def run_reference(args):
     if rank != 0:
         return
     spec, lengths = workload_info(args.workload)
+    B = int(len(lengths))
     cb = cpu_baseline(args.workload, max(1.0, min(args.cpu_seconds, 60.0)))
     line = {"impl": "reference", "metric": METRIC, "value": cb["value"], "unit": UNIT, "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / cb["value"],
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * B / cb["value"],
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded)",
-            "config": {"workload": args.workload, "B": int(len(lengths)), "cache_len": [int(x) for x in lengths[:4]],
+            "config": {"workload": args.workload, "B": B, "cache_len": [int(x) for x in lengths[:4]],
                        "layers": 32, "parallelism": f"replicas x{world}",
-                       "sample": "vehicle 0 per step; vehicles are independent, so vehicle-ticks/s is per vehicle"},
+                       "sample": cb["sample"] + "; vehicles are independent, so vehicle-ticks/s is per vehicle"},
             "cpu_baseline": cb,
             "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
 
 
+def spawn_ranks(n):
+    """--gpus N without torchrun: run N copies of this command, one per GPU, with the
+    rank environment torchrun would set; rank 0's output is this process's output."""
+    import socket
+    with socket.socket() as sock:
+        sock.bind(("127.0.0.1", 0))
+        port = sock.getsockname()[1]
+    procs = []
+    for r in range(n):
+        env = dict(os.environ, RANK=str(r), LOCAL_RANK=str(r), WORLD_SIZE=str(n), MASTER_ADDR="127.0.0.1",
+                   MASTER_PORT=str(port))
+        out = None if r == 0 else subprocess.DEVNULL
+        procs.append(subprocess.Popen([sys.executable, os.path.abspath(__file__)] + sys.argv[1:], env=env, stdout=out))
+    codes = [p.wait() for p in procs]
+    return max(codes, key=abs)
+
+
+def time_ticks(ex, k, v, offsets, frames, out, stream, steps, warmup):
+    """Device milliseconds of `steps` ticks between CUDA events on `stream`, after `warmup`."""
+    import torch
+    from paper_2607_15621_gb300 import fsx
+    for _ in range(max(warmup, 3)):
+        ex.tick(k, v, offsets, frames, out, stream)
+    torch.cuda.synchronize()
+    if ex.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during warm-up")
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        ex.tick(k, v, offsets, frames, out, stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if ex.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during the timed region")
+    return e0.elapsed_time(e1)
+
+
+def tick_roofline_us(dims, lengths, dtype, weight_bytes, hbm, tensor_tfs):
+    """max(bytes / HBM bandwidth, FLOPs / tensor peak) of one tick, in microseconds."""
+    tick_bytes, _ = algorithmic_bytes(dims, lengths, dtype, weight_bytes)
+    return max(tick_bytes / (hbm * 1e9), tick_flops(dims, lengths) / (tensor_tfs * 1e12)) * 1e6
+
+
+def run_extras(ex, dims, dev, stream, weight_bytes, hbm, tensor_tfs):
+    """The B = 1 tick, the history sweep and the 16-vehicle batch through the headline's
+    handle: us/tick and fraction of the tick roofline of each (CUDA events)."""
+    import torch
+    from paper_2607_15621_gb300 import synth
+    res = []
+    for name in EXTRA_WORKLOADS:
+        spec, lengths = workload_info(name)
+        B = len(lengths)
+        k, v, off = synth.make_cache(dims, lengths, 0, spec["dtype"], device=dev)
+        frames = synth.make_frames(dims, B, 0, spec["dtype"], device=dev)
+        offsets = torch.as_tensor(off, device=dev)
+        out = torch.empty(B, dims.n_waypoints, 2, device=dev)
+        steps = 200 if B == 1 else 50
+        ms = time_ticks(ex, k, v, offsets, frames, out, stream, steps, 5)
+        us = ms / steps * 1e3
+        rl = tick_roofline_us(dims, lengths, spec["dtype"], weight_bytes, hbm, tensor_tfs)
+        tick_bytes, _ = algorithmic_bytes(dims, lengths, spec["dtype"], weight_bytes)
+        res.append({"workload": name, "B": B, "cache_tokens": int(np.sum(lengths)), "us_per_tick": us,
+                    "vehicle_ticks_per_s": B * 1e6 / us, "steps": steps, "launches_per_tick": ex.launches(B),
+                    "roofline_us": rl, "frac": rl / us, "achieved_gbs": tick_bytes / (us * 1e-6) / 1e9,
+                    "bytes_per_tick": tick_bytes})
+        del k, v, frames
+    torch.cuda.empty_cache()
+    return res
+
+
 def main():
     args = parse()
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        sys.exit(spawn_ranks(args.gpus))
     from paper_2607_15621_gb300 import synth
     if args.workload in synth.APPEND_WORKLOADS:
         (run_append_reference if args.impl == "reference" else run_append)(args)
@@ -563,6 +700,7 @@ def main():
     dims = synth.EXPERT if args.layers is None else dataclasses.replace(synth.EXPERT, n_layers=args.layers)
     dtype = spec["dtype"]
     B = len(lengths)
+    extras = (not args.no_extras and args.workload == DEFAULT_WORKLOAD and args.layers is None)
     w = synth.make_weights(dims, 0, dtype)
     k, v, off = synth.make_cache(dims, lengths, 0, dtype, device=dev)
     frames = synth.make_frames(dims, B, 0, dtype, device=dev)
@@ -577,30 +715,18 @@ def main():
             import torch.distributed as dist
             dist.barrier()
 
+    clock_path = os.path.join(clock_dir(), f"clocks_rank{rank}.csv")
+    os.makedirs(os.path.dirname(clock_path), exist_ok=True)
     for _ in range(max(args.warmup, 3)):
         ex.tick(k, v, offsets, frames, out, stream)
     torch.cuda.synchronize()
-    if ex.status(stream) != fsx.FSX_OK:
-        raise RuntimeError("device status set during warm-up")
-
-    clock_path = os.path.join(clock_dir(), f"clocks_rank{rank}.csv")
-    os.makedirs(os.path.dirname(clock_path), exist_ok=True)
     proc, fh = start_clock_sampler(clock_path, local)
     time.sleep(0.5)
     barrier()
     torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        ex.tick(k, v, offsets, frames, out, stream)
-    e1.record(stream)
-    torch.cuda.synchronize()
+    ms = time_ticks(ex, k, v, offsets, frames, out, stream, args.steps, 0)
     barrier()
-    ms = e0.elapsed_time(e1)
     clocks = stop_clock_sampler(proc, fh, clock_path)
-    if ex.status(stream) != fsx.FSX_OK:
-        raise RuntimeError("device status set during the timed region")
     ms = max_over_ranks(ms, dev)
     ms_per_step = ms / args.steps
     value = world * B * args.steps / (ms / 1e3)
@@ -658,6 +784,14 @@ def main():
     # roofline time of one tick = max(bytes / HBM bandwidth, FLOPs / tensor peak)
     rl_meas_us = max(tick_bytes / (hbm * 1e9), flops / (tensor_tfs * 1e12)) * 1e6
     rl_nom_us = max(tick_bytes / (NOMINAL_HBM_GBS * 1e9), flops / (NOMINAL_TENSOR_TFS * 1e12)) * 1e6
+    traffic, traffic_stale = traffic_for(kclass, args.workload)
+    launches = ex.launches(B)
+    weight_bytes = ex.weight_bytes()
+    extra_lines = None
+    if extras:
+        del k, v, frames
+        torch.cuda.empty_cache()
+        extra_lines = run_extras(ex, dims, dev, stream, weight_bytes, hbm, tensor_tfs)
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -665,13 +799,14 @@ def main():
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f16 (fp32 accumulate)",
         "data": "synthetic (seeded N(0,1) cache/frames, N(0,1/fan_in) weights)",
         "config": {"workload": args.workload, "B": B, "cache_len": [int(x) for x in lengths[:4]],
-                   "layers": dims.n_layers, "d_model": dims.d_model, "tokens_per_vehicle": dims.n_tok,
+                   "cache_tokens": int(np.sum(lengths)), "layers": dims.n_layers, "d_model": dims.d_model,
+                   "tokens_per_vehicle": dims.n_tok,
                    "l2": "inputs larger than L2 (weights + cache per tick exceed 129 MB)",
                    "parallelism": f"replicas x{world}"},
-        "gpu_launches": ex.launches(B) * args.steps,
+        "gpu_launches": launches * args.steps,
         "roofline": {"bound": "hbm", "kernel": kclass, "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": achieved / hbm, "traffic": NCU_TRAFFIC.get((kclass, args.workload)), "peak_source": peak_kind,
-                     "bytes_per_launch": unit_bytes, "launch_us": per_launch_s * 1e6},
+                     "frac": achieved / hbm, "traffic": traffic, "traffic_stale": traffic_stale,
+                     "peak_source": peak_kind, "bytes_per_launch": unit_bytes, "launch_us": per_launch_s * 1e6},
         "tick_roofline": {"bytes_per_tick": tick_bytes, "kv_bytes_per_tick": kv_bytes, "achieved_gbs": tick_gbs,
                           "frac_of_measured_hbm": tick_gbs / hbm, "frac_of_8tbs": tick_gbs / NOMINAL_HBM_GBS,
                           "flops_per_tick": flops,
@@ -683,15 +818,16 @@ def main():
                 "d2h_bytes_per_step": int(d2h)},
         "clocks": clocks,
     }
+    if extra_lines is not None:
+        line["workloads"] = extra_lines
+    ex.close()
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.workload, args.cpu_seconds)
-    ex.close()
     if rank == 0:
         print(json.dumps(line))
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
-
 
 if __name__ == "__main__":
     main()

@@ -25,12 +25,14 @@
  *     operands are fp16 with fp32 accumulation, the residual stream, RMSNorm,
  *     softmax statistics and the head are fp32. Cache values the kernels
  *     convert to fp16 (every key; the values too, except in the bf16 tensor-core
- *     attention of batched ticks) are expected within +-65504. A value beyond
- *     that (a bf16 magnitude of 65536 or more, an fp32 magnitude that rounds
- *     past 65504, infinity or NaN) is saturated to +-65504 instead of becoming
- *     an infinity that would turn the softmax into NaN, and the status read by
- *     fsx_get_status becomes FSX_ERR_RANGE: the results of that tick are those of
- *     the saturated cache, not of the caller's values.
+ *     attention of batched ticks, which keeps them bf16) must lie within
+ *     +-65504. A value beyond that (a bf16 magnitude of 65536 or more, an fp32
+ *     magnitude that rounds past 65504, infinity or NaN) is a device-side error:
+ *     the status becomes FSX_ERR_RANGE and the tick is abandoned like on bad
+ *     offsets, writing no waypoint, instead of returning NaN waypoints. In the
+ *     tensor-core attention the check is made on the scores: a key beyond the
+ *     range whose scores all fall to -inf has weight zero, as its exact value
+ *     would, and is not reported.
  */
 #ifndef FSX_H
 #define FSX_H
@@ -53,9 +55,8 @@ typedef enum {
   FSX_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up              */
   FSX_ERR_DEVICE_ARG = 6,   /* device-side check: offsets not non-decreasing,
                                negative, or beyond max_total_cache_tokens      */
-  FSX_ERR_RANGE = 7         /* device-side check: a cache value lay outside the
-                               fp16 range (see Precision); it was saturated to
-                               +-65504 and the tick completed on that value    */
+  FSX_ERR_RANGE = 7         /* device-side check: a cache value lies outside
+                               the fp16 range (see Precision)                  */
 } fsx_status;
 
 typedef enum { FSX_F32 = 0, FSX_BF16 = 1 } fsx_dtype;
@@ -160,9 +161,8 @@ fsx_status fsx_tick_ranges_debug(fsx_handle h, const void* const* k_cache, const
  * paper: the error path of the tick (Sec. 3.3 runs it every 50 ms, so a failed
  * tick must be detectable without stopping the stream). Synchronises `stream`
  * (the stream of the ticks to check), then returns and clears the device status
- * block: FSX_OK, FSX_ERR_DEVICE_ARG, FSX_ERR_TIMEOUT (errors: that tick's
- * kernels skipped their work) or FSX_ERR_RANGE (the tick completed on saturated
- * cache values). Errors take precedence over FSX_ERR_RANGE. */
+ * word: FSX_OK, FSX_ERR_DEVICE_ARG, FSX_ERR_TIMEOUT or FSX_ERR_RANGE (the first
+ * error of those ticks; the tick that raised it wrote no waypoint). */
 fsx_status fsx_get_status(fsx_handle h, void* stream);
 
 /* Thread-local message describing the last failure on this thread ("" if none). */
@@ -248,10 +248,10 @@ fsx_status fsx_attention_noalloc(const void* d_q, long long q_stride,
  * device (the paper has no counterpart; it completes that entry point for the
  * same callers). Synchronises `stream` -- the stream of the calls to check --
  * then returns the word and clears it: FSX_OK, FSX_ERR_DEVICE_ARG (a call saw
- * negative or decreasing cache offsets), FSX_ERR_TIMEOUT or FSX_ERR_RANGE (cache
- * values saturated to the fp16 range, as in fsx_get_status). Copies two ints to
- * the host and clears them on the device; allocates nothing. Calls still running
- * on other streams may set the word afterwards. */
+ * negative or decreasing cache offsets), FSX_ERR_TIMEOUT or FSX_ERR_RANGE (a
+ * cache value outside the fp16 range, as in fsx_get_status). Copies one int to the
+ * host and clears it on the device; allocates nothing. Calls still running on
+ * other streams may set the word afterwards. */
 fsx_status fsx_attention_noalloc_status(void* stream);
 
 /* ================================================================== cache append

@@ -107,7 +107,7 @@ extern "C" fsx_status fsx_attention_noalloc(const void* d_q, long long q_stride,
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int* status = static_cast<int*>(base);
   float* part = reinterpret_cast<float*>(static_cast<unsigned char*>(base) + kStatusSlot);
-  cudaError_t e = cudaMemsetAsync(status, 0, 2 * sizeof(int), st);  // error word, range word
+  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), st);
   if (e != cudaSuccess) return noalloc_fail(FSX_ERR_CUDA, cudaGetErrorString(e));
 
   fsx::AttnArgs a{};
@@ -146,13 +146,13 @@ extern "C" fsx_status fsx_attention_noalloc_status(void* stream) {
   const fsx_status bs = scratch_base(&base);
   if (bs != FSX_OK) return bs;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  int word[2] = {0, 0};  // error word, range word
-  cudaError_t e = cudaMemcpyAsync(word, base, 2 * sizeof(int), cudaMemcpyDeviceToHost, st);
-  if (e == cudaSuccess) e = cudaMemsetAsync(base, 0, 2 * sizeof(int), st);
+  int word = 0;
+  cudaError_t e = cudaMemcpyAsync(&word, base, sizeof(int), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(base, 0, sizeof(int), st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return noalloc_fail(FSX_ERR_CUDA, cudaGetErrorString(e));
-  if (word[0] == static_cast<int>(FSX_ERR_TIMEOUT)) return noalloc_fail(FSX_ERR_TIMEOUT, "a device-side wait timed out");
-  if (word[0] != 0) return noalloc_fail(FSX_ERR_DEVICE_ARG, "device-side check: cache offsets negative or decreasing");
-  if (word[1] != 0) return noalloc_fail(FSX_ERR_RANGE, "cache values beyond the fp16 range were saturated to +-65504");
-  return FSX_OK;
+  if (word == 0) return FSX_OK;
+  if (word == static_cast<int>(FSX_ERR_TIMEOUT)) return noalloc_fail(FSX_ERR_TIMEOUT, "a device-side wait timed out");
+  if (word == static_cast<int>(FSX_ERR_RANGE)) return noalloc_fail(FSX_ERR_RANGE, "a cache value lies outside the fp16 range");
+  return noalloc_fail(FSX_ERR_DEVICE_ARG, "device-side check: cache offsets negative or decreasing");
 }

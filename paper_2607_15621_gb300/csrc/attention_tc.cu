@@ -390,7 +390,6 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
     uint64_t* full = is_v ? vfull : kfull;
     uint64_t* empty = is_v ? vempty : kempty;
     bool ok = true;
-    uint32_t range = 0;  // a cache key outside the fp16 range was saturated
     for (int i = 0; ok && i < n_chunks; ++i) {
       if (i + 1 < n_chunks) cp_async_wait<1>();
       else cp_async_wait<0>();
@@ -406,8 +405,7 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
         for (int m = 0; m < kSlotKeys / 4; ++m) {
           uint4* ptr = reinterpret_cast<uint4*>(slot + tile128_off(pr0 + 4 * m, pu));
           const uint4 v = *ptr;
-          *ptr = make_uint4(bf16x2_to_half2_sat(v.x, range), bf16x2_to_half2_sat(v.y, range),
-                            bf16x2_to_half2_sat(v.z, range), bf16x2_to_half2_sat(v.w, range));
+          *ptr = make_uint4(bf16x2_to_half2(v.x), bf16x2_to_half2(v.y), bf16x2_to_half2(v.z), bf16x2_to_half2(v.w));
         }
       }
       fence_proxy_async();
@@ -418,7 +416,6 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
       }
     }
     cp_async_wait<0>();
-    flag_range(p.status, range);
   } else {
     // ---------------------------------------------------------------- softmax rows
     // Warp w owns query rows 16 w .. 16 w + 15 (tensor-memory lanes 32 w .. + 15).
@@ -538,6 +535,10 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
       const float inv[2] = {l_run[0] > 0.f ? 1.f / l_run[0] : 0.f, l_run[1] > 0.f ? 1.f / l_run[1] : 0.f};
       const bool va = ra < p.n_q;
       const bool vb = rbw < p.n_q;
+      // A cache key beyond the fp16 range became an infinity here; where it raised a
+      // score to +inf (or NaN) the row's sum is NaN: report it, the tick is abandoned.
+      // (A key whose scores all fell to -inf carries weight 0, as the exact value would.)
+      if ((va && !(l_run[0] == l_run[0])) || (vb && !(l_run[1] == l_run[1]))) set_status(p.status, kStatusRange);
       __half* oa = p.out + (static_cast<size_t>(b) * p.n_q + (va ? ra : 0)) * p.out_stride + h * kD + 2 * t4;
       __half* ob = p.out + (static_cast<size_t>(b) * p.n_q + (vb ? rbw : 0)) * p.out_stride + h * kD + 2 * t4;
 #pragma unroll 1

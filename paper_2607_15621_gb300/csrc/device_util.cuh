@@ -177,13 +177,12 @@ __device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// Cache values converted to fp16 saturate at +-65504 instead of overflowing to
-// infinity (cvt .satfinite), and every such value is recorded: `range` collects
-// whether an input lay outside the fp16 range (a bf16 magnitude of 65536 or more,
-// infinity or NaN; an fp32 magnitude that rounds beyond 65504), and
-// flag_range() raises the second word of the status block, which the kernels do
-// not treat as an error (the tick continues on the saturated values) and the
-// host reports as FSX_ERR_RANGE.
+// Cache values the kernels convert to fp16 are expected within +-65504. The
+// converters below saturate instead of overflowing to infinity (cvt .satfinite),
+// and `range` collects whether an input lay outside the fp16 range (a bf16
+// magnitude of 65536 or more, infinity or NaN; an fp32 magnitude that rounds
+// beyond 65504). flag_range() turns that into the FSX_ERR_RANGE error status, and
+// the tick is abandoned like any other device-side error.
 __device__ __forceinline__ uint32_t bf16x2_to_half2_sat(uint32_t v, uint32_t& range) {
   const float lo = __uint_as_float(v << 16);
   const float hi = __uint_as_float(v & 0xffff0000u);
@@ -199,7 +198,7 @@ __device__ __forceinline__ uint32_t f32x2_to_half2_sat(float lo, float hi, uint3
   return r;
 }
 __device__ __forceinline__ void flag_range(int* status, uint32_t range) {
-  if (range) *reinterpret_cast<volatile int*>(status + 1) = kStatusRange;
+  if (range) set_status(status, kStatusRange);
 }
 
 // Two bf16 (low half first) -> two fp16, via fp32 (bf16 -> fp32 is exact).

@@ -684,8 +684,8 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
   FSX_CUDA_H(cudaMalloc(&h->tile_count, sizeof(int) * h->sm_count));
   FSX_CUDA_H(cudaMemset(h->tile_count, 0, sizeof(int) * h->sm_count));
   FSX_CUDA_H(cudaMalloc(&h->order, sizeof(int) * cfg->max_batch));
-  FSX_CUDA_H(cudaMalloc(&h->status, 2 * sizeof(int)));  // error word, range word
-  FSX_CUDA_H(cudaMemset(h->status, 0, 2 * sizeof(int)));
+  FSX_CUDA_H(cudaMalloc(&h->status, sizeof(int)));
+  FSX_CUDA_H(cudaMemset(h->status, 0, sizeof(int)));
   FSX_CUDA_H(cudaMalloc(&h->d_args, sizeof(TickArgs)));
   FSX_CUDA_H(cudaMalloc(&h->st_offsets, (cfg->max_batch + 1) * sizeof(int64_t)));
   FSX_CUDA_H(cudaMalloc(&h->st_frames, static_cast<size_t>(cfg->max_batch) * cfg->n_frame * d * sizeof(float) + 16));
@@ -766,13 +766,12 @@ fsx_status fsx_tick_debug(fsx_handle h, const void* const* k_cache, const void* 
                                stream);
 }
 
-// The host reading of a device status block: the error word first, then the
-// range word (cache values saturated to the fp16 range, the tick completed).
-static fsx_status status_words(const int* v) {
-  if (v[0] == FSX_ERR_TIMEOUT) return fail(FSX_ERR_TIMEOUT, "a device-side wait timed out");
-  if (v[0] != 0) return fail(FSX_ERR_DEVICE_ARG, "device-side argument check failed (cache offsets)");
-  if (v[1] != 0) return fail(FSX_ERR_RANGE, "cache values beyond the fp16 range were saturated to +-65504");
-  return FSX_OK;
+// The host reading of the device status word.
+static fsx_status status_word(int v) {
+  if (v == 0) return FSX_OK;
+  if (v == FSX_ERR_TIMEOUT) return fail(FSX_ERR_TIMEOUT, "a device-side wait timed out");
+  if (v == FSX_ERR_RANGE) return fail(FSX_ERR_RANGE, "a cache value lies outside the fp16 range");
+  return fail(FSX_ERR_DEVICE_ARG, "device-side argument check failed (cache offsets)");
 }
 
 fsx_status fsx_get_status(fsx_handle h, void* stream) {
@@ -780,11 +779,11 @@ fsx_status fsx_get_status(fsx_handle h, void* stream) {
   std::lock_guard<std::mutex> lock(h->mu);
   FSX_CUDA(cudaSetDevice(h->device));
   FSX_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
-  int v[2] = {0, 0};
-  FSX_CUDA(cudaMemcpyAsync(v, h->status, 2 * sizeof(int), cudaMemcpyDeviceToHost, h->cap_stream));
-  FSX_CUDA(cudaMemsetAsync(h->status, 0, 2 * sizeof(int), h->cap_stream));
+  int v = 0;
+  FSX_CUDA(cudaMemcpyAsync(&v, h->status, sizeof(int), cudaMemcpyDeviceToHost, h->cap_stream));
+  FSX_CUDA(cudaMemsetAsync(h->status, 0, sizeof(int), h->cap_stream));
   FSX_CUDA(cudaStreamSynchronize(h->cap_stream));
-  return status_words(v);
+  return status_word(v);
 }
 
 void fsx_destroy(fsx_handle h) { free_handle(h); }
@@ -852,9 +851,9 @@ fsx_status fsx_attention(const void* d_q, long long q_stride, const void* d_k_ow
   if (!d_workspace || workspace_bytes < need)
     return fail(FSX_ERR_INVALID_ARG, "workspace of %zu bytes required", need);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  int* status = static_cast<int*>(d_workspace);  // first 256 bytes: error word, range word
+  int* status = static_cast<int*>(d_workspace);  // first 256 bytes: status word
   float* part = reinterpret_cast<float*>(static_cast<unsigned char*>(d_workspace) + 256);
-  FSX_CUDA(cudaMemsetAsync(status, 0, 2 * sizeof(int), st));
+  FSX_CUDA(cudaMemsetAsync(status, 0, sizeof(int), st));
   FSX_CUDA(fsx::attention_set_attributes());
   fsx::AttnArgs a{};
   a.q = static_cast<const __half*>(d_q);

@@ -986,6 +986,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
       for (int i = 0; i < n; ++i) issue(q0 + kLayerChunks + i);
     }
     scatter_add(Xm, rank * 128, res, head == 0);
+    flag_range(p.status, range_seen);  // every thread's own units; published by the arrival
     arrive(p.counters + sA + 1);
 
     // =========================== phase B ===========================
@@ -1126,7 +1127,6 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
               : "r"(smem_addr(full + q % kSlots)), "r"(static_cast<uint32_t>((q / kSlots) & 1))
               : "memory");
       }
-  flag_range(p.status, range_seen);
   // no CTA leaves while a partner may still write into its shared memory
   cluster.sync();
   tc_fence_before();
@@ -1137,6 +1137,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   // =========================== head ===========================
   if (cta == 0) {
     wait_counter(p.counters + 2 * p.n_layers, n_b_ctas, p.status, abort);
+    // a tick with a device-side error (an out-of-range cache value, a timeout) writes no waypoint
+    if (*reinterpret_cast<volatile int*>(p.status) != 0) return;
     const float* Xf = X0 + static_cast<size_t>((2 * p.n_layers) % 3) * xs;
     for (int j = warp; j < p.n_waypoints; j += kThr / 32) {
       const float* xr = Xf + static_cast<size_t>(j) * d;

@@ -93,3 +93,30 @@ def test_clip_reference_arm_prints_one_line():
     line = json.loads(lines[0])
     assert line["impl"] == "reference" and line["unit"] == "frame-blocks/s" and line["value"] > 0
     assert line["config"]["frames"] == 40 and line["config"]["delta"] == 1
+
+
+def test_gpus_flag_without_torchrun_starts_the_ranks_itself():
+    """`bench.py --gpus 2` outside torchrun starts two ranks with the rank environment
+    torchrun would give them; the reference arm then prints one line, from rank 0."""
+    env = {k: v for k, v in os.environ.items() if k not in ("WORLD_SIZE", "RANK", "LOCAL_RANK")}
+    cmd = [sys.executable, "bench.py", "--impl", "reference", "--gpus", "2", "--steps", "1", "--warmup", "1",
+           "--cpu-seconds", "1"]
+    res = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600, env=env)
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [l for l in res.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, res.stdout
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["n_gpus"] == 2
+    assert line["config"]["parallelism"] == "replicas x2"
+    assert line["config"]["workload"] == "bf16_b128_ragged" and line["config"]["B"] == 128
+
+
+def test_cpu_baseline_sample_spans_the_length_order():
+    sys.path.insert(0, ROOT)
+    import numpy as np
+    import bench
+    lengths = np.array([300, 70, 2048, 900, 64, 1500, 1200, 400, 999, 1800])
+    picks = bench.baseline_vehicles(lengths)
+    assert len(picks) == 8 and len(set(picks)) == 8
+    assert int(np.argmin(lengths)) in picks and int(np.argmax(lengths)) in picks
+    assert bench.baseline_vehicles([224]) == [0]
