@@ -18,6 +18,8 @@ exceed the 129 MB L2, so no flush is needed between ticks.
 The workload `clip_j40_delta1` times the staleness-masked forward over a 40-frame
 clip (Sec. 3.2: every frame block over the cache prefix ending one frame earlier,
 all blocks in one tick over explicit row ranges); value = frame-blocks/s.
+The workload `paper_b1_l224` times the paper's own ten-token layout (state token,
+four visual tokens, five queries, two-layer head; Sec. 3.1) at B = 1, L = 224.
 The workload `append_b1_l224` instead times the backbone's incremental cache
 append (one call = n_new = 4 tokens through the 32-layer, 4096-wide backbone
 for one vehicle with 224 cached tokens); value = vehicle-appends/s.
@@ -583,6 +585,148 @@ def run_clip(args):
         dist.destroy_process_group()
 
 
+PAPER_METRIC = "vehicle-ticks/s (1e6 / us-per-tick x B) of the ten-token expert tick (state token, 4 visual, 5 queries)"
+
+
+def paper_inputs(args, device):
+    from paper_2607_15621_gb300 import synth
+    spec = synth.PAPER_WORKLOADS[args.workload]
+    dims = dataclasses.replace(synth.EXPERT, n_action=5, n_frame=5)
+    if args.layers is not None:
+        dims = dataclasses.replace(dims, n_layers=args.layers)
+    B, L = spec["batch"], spec["length"]
+    w = synth.make_paper_weights(dims, 0, "bf16")
+    k, v, off = synth.make_cache(dims, [L] * B, 0, "bf16", device=device)
+    visual, state = synth.make_paper_inputs(dims, B, 0, "bf16", device=device)
+    return dims, w, k, v, off, visual, state, B, L
+
+
+def run_paper_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from oracle import paper_tokens_oracle
+    dims, w, k, v, off, visual, state, B, L = paper_inputs(args, "cpu")
+    kn = [t.float().numpy() for t in k]
+    vn = [t.float().numpy() for t in v]
+    vis = visual[:1].double().numpy()
+    st = state[:1].double().numpy()
+    lo, hi = int(off[0]), int(off[1])
+    seconds = max(1.0, min(args.cpu_seconds, 60.0))
+    n, t0 = 0, time.perf_counter()
+    while True:
+        paper_tokens_oracle.expert_tick_paper_tokens(w, [t[lo:hi] for t in kn], [t[lo:hi] for t in vn],
+                                                     np.array([0, hi - lo]), vis, st, dims.n_heads, dims.head_dim)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or n >= 1000:
+            break
+    cb = {"value": n / el, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+          "sample": f"{n} full {dims.n_layers}-layer fp64 ten-token ticks of vehicle 0 of {args.workload} (L={L}) "
+                    f"in {el:.1f} s"}
+    line = {"impl": "reference", "metric": PAPER_METRIC, "value": cb["value"], "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * B / cb["value"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded)",
+            "config": {"workload": args.workload, "B": B, "cache_len": L, "layers": dims.n_layers,
+                       "tokens_per_vehicle": 10, "parallelism": f"replicas x{world}",
+                       "sample": "vehicle 0 per step; vehicles are independent"},
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def run_paper(args):
+    """The ten-token tick on the GPU: CUDA events around K ticks (state MLP, layer stack,
+    two-layer head), inputs resident in HBM; e2e with the visual tokens and ego state
+    copied in from pinned host memory and the waypoints read back every tick."""
+    import torch
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2607_15621_gb300 import fsx
+    dims, w, k, v, off, visual, state, B, L = paper_inputs(args, dev)
+    offsets = torch.as_tensor(off, device=dev)
+    out = torch.empty(B, 5, 2, device=dev)
+    ex = fsx.PaperExpert(dims, w, B, int(off[-1]), "bf16", "bf16", device=local)
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(max(args.warmup, 3)):
+        ex.paper_tick(k, v, offsets, visual, state, out, stream)
+    torch.cuda.synchronize()
+    if ex.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during warm-up")
+    clock_path = os.path.join(clock_dir(), f"clocks_rank{rank}.csv")
+    os.makedirs(os.path.dirname(clock_path), exist_ok=True)
+    proc, fh = start_clock_sampler(clock_path, local)
+    time.sleep(0.5)
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        ex.paper_tick(k, v, offsets, visual, state, out, stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    ms = max_over_ranks(e0.elapsed_time(e1), dev)
+    clocks = stop_clock_sampler(proc, fh, clock_path)
+    if ex.status(stream) != fsx.FSX_OK:
+        raise RuntimeError("device status set during the timed region")
+    ms_per_step = ms / args.steps
+    vis_h = visual.cpu().pin_memory()
+    st_h = state.cpu().pin_memory()
+    out_h = torch.empty(B, 5, 2).pin_memory()
+    e2e_steps = max(1, args.steps // 2)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        visual.copy_(vis_h, non_blocking=True)
+        state.copy_(st_h, non_blocking=True)
+        ex.paper_tick(k, v, offsets, visual, state, out, stream)
+        out_h.copy_(out, non_blocking=True)
+        stream.synchronize()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
+    hbm, tensor_tfs, peak_kind = peaks()
+    tick_bytes, _ = algorithmic_bytes(dims, [L] * B, "bf16", ex.weight_bytes())
+    flops = tick_flops(dims, [L] * B)
+    rl_us = max(tick_bytes / (hbm * 1e9), flops / (tensor_tfs * 1e12)) * 1e6
+    achieved = tick_bytes / (ms_per_step / 1e3) / 1e9
+    line = {
+        "metric": PAPER_METRIC, "value": world * B / (ms_per_step / 1e3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_per_step,
+        "us_per_tick": ms_per_step * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f16 (fp32 accumulate)", "data": "synthetic (seeded N(0,1) cache/visual/state, N(0,1/fan_in) weights)",
+        "config": {"workload": args.workload, "B": B, "cache_len": L, "layers": dims.n_layers, "tokens_per_vehicle": 10,
+                   "l2": "inputs larger than L2 (the expert weights exceed 129 MB)",
+                   "parallelism": f"replicas x{world}"},
+        "gpu_launches": (1 + ex.launches(B)) * args.steps,
+        "roofline": {"bound": "hbm", "kernel": "ten-token tick (state MLP, tick, head)", "achieved": achieved,
+                     "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": None, "peak_source": peak_kind,
+                     "bytes_per_launch": tick_bytes, "launch_us": ms_per_step * 1e3, "flops_per_tick": flops,
+                     "roofline_us": rl_us, "frac_of_tick_roofline": rl_us / (ms_per_step * 1e3)},
+        "e2e": {"value": world * B * e2e_steps / e2e_s, "unit": UNIT,
+                "h2d_bytes_per_step": int(vis_h.numel() * vis_h.element_size() + st_h.numel() * 4),
+                "d2h_bytes_per_step": int(out_h.numel() * 4)},
+        "clocks": clocks,
+    }
+    ex.close()
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def run_reference(args):
     world, rank, _ = dist_env()
     if rank != 0:
@@ -684,6 +828,9 @@ def main():
     if args.workload in synth.CLIP_WORKLOADS:
         (run_clip_reference if args.impl == "reference" else run_clip)(args)
         return
+    if args.workload in synth.PAPER_WORKLOADS:
+        (run_paper_reference if args.impl == "reference" else run_paper)(args)
+        return
     if args.impl == "reference":
         run_reference(args)
         return
@@ -765,17 +912,23 @@ def main():
     ex.set_kernel_timing(False, kclass)
     per_launch_s = statistics.mean(kt_ms) / kt_n / 1e3
     d, hd, f = dims.d_model, dims.hd, dims.d_ff
-    M = B * dims.n_tok
-    unit_bytes = {  # algorithmic bytes of one launch (one layer): weights + activations in/out
-        "qkv": 3 * hd * d * 2 + M * d * 4 + M * 3 * hd * 2,
-        "out_proj": d * hd * 2 + M * hd * 2 + 2 * M * d * 4,
-        "gate_up": 2 * f * d * 2 + M * d * 4 + M * f * 2,
-        "down": d * f * 2 + M * f * 2 + 2 * M * d * 4,
-        "attention": int(np.sum(lengths)) * 2 * hd * (2 if dtype == "bf16" else 4) + M * 3 * hd * 2 + M * hd * 2,
+    # a batch may run as several chains (vehicle groups), each with its own launch of a
+    # kernel class per layer: average algorithmic bytes of one launch = the class's bytes
+    # per tick / its launches per tick
+    chains = max(1, kt_n // dims.n_layers) if kclass != "persistent" else 1
+    Mc = B * dims.n_tok / chains  # token rows of one chain
+    unit_bytes = {  # algorithmic bytes of one launch (one layer of one chain): weights + activations in/out
+        "qkv": 3 * hd * d * 2 + Mc * d * 4 + Mc * 3 * hd * 2,
+        "out_proj": d * hd * 2 + Mc * hd * 2 + 2 * Mc * d * 4,
+        "gate_up": 2 * f * d * 2 + Mc * d * 4 + Mc * f * 2,
+        "down": d * f * 2 + Mc * f * 2 + 2 * Mc * d * 4,
+        "attention": (int(np.sum(lengths)) * 2 * hd * (2 if dtype == "bf16" else 4)) / chains + Mc * 3 * hd * 2
+                     + Mc * hd * 2,
         "persistent": None,
     }[kclass]
     if unit_bytes is None:  # one launch = the whole tick: weights + cache rows
         unit_bytes = algorithmic_bytes(dims, lengths, dtype, ex.weight_bytes())[0]
+    unit_bytes = int(unit_bytes)
     hbm, tensor_tfs, peak_kind = peaks()
     achieved = unit_bytes / per_launch_s / 1e9
     tick_bytes, kv_bytes = algorithmic_bytes(dims, lengths, dtype, ex.weight_bytes())
@@ -806,7 +959,8 @@ def main():
         "gpu_launches": launches * args.steps,
         "roofline": {"bound": "hbm", "kernel": kclass, "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm, "traffic": traffic, "traffic_stale": traffic_stale,
-                     "peak_source": peak_kind, "bytes_per_launch": unit_bytes, "launch_us": per_launch_s * 1e6},
+                     "peak_source": peak_kind, "bytes_per_launch": unit_bytes, "launch_us": per_launch_s * 1e6,
+                     "launches_per_tick": kt_n},
         "tick_roofline": {"bytes_per_tick": tick_bytes, "kv_bytes_per_tick": kv_bytes, "achieved_gbs": tick_gbs,
                           "frac_of_measured_hbm": tick_gbs / hbm, "frac_of_8tbs": tick_gbs / NOMINAL_HBM_GBS,
                           "flops_per_tick": flops,

@@ -254,6 +254,60 @@ fsx_status fsx_attention_noalloc(const void* d_q, long long q_stride,
  * other streams may set the word afterwards. */
 fsx_status fsx_attention_noalloc_status(void* stream);
 
+/* ============================================================ the paper's ten-token expert
+ * Sec. 3.1 gives the expert ten tokens per vehicle and frame: one state token that
+ * embeds the ego state -- the previous five predicted waypoints (x, y), the previous
+ * control triplet (throttle, steer, brake), the current speed and the target point
+ * (x, y), 16 values in that order -- the current frame's four visual tokens, and five
+ * learned waypoint queries; a two-layer head decodes the five query outputs into five
+ * (x, y) waypoints. The layer stack is the tick above.
+ *   state token  t = W_s2 silu(W_s1 s + b_s1) + b_s2
+ *   tokens       X = [t ; V (4 visual tokens) ; E_q (5 queries)] + P_pos
+ *   waypoint i   w_i = W_h2 silu(W_h1 RMSNorm(X_{5+i}; g_f) + b_h1) + b_h2
+ * Host fp32 weights, every matrix row-major [out_features, in_features], copied at
+ * create; the layer weights are those of fsx_weights. */
+typedef struct {
+  const float* state_w1;   /* [d, 16]    state MLP, first layer    */
+  const float* state_b1;   /* [d]                                  */
+  const float* state_w2;   /* [d, d]     state MLP, second layer   */
+  const float* state_b2;   /* [d]                                  */
+  const float* query_emb;  /* [5, d]     learned waypoint queries   */
+  const float* pos_emb;    /* [10, d]    positions: state, visual 0-3, queries 0-4 */
+  const float* attn_norm;  /* [n_layers, d]   as fsx_weights       */
+  const float* wq;         /* [n_layers, n_heads*head_dim, d]      */
+  const float* wk;
+  const float* wv;
+  const float* wo;         /* [n_layers, d, n_heads*head_dim]      */
+  const float* mlp_norm;   /* [n_layers, d]                        */
+  const float* w_gate;     /* [n_layers, d_ff, d]                  */
+  const float* w_up;
+  const float* w_down;     /* [n_layers, d, d_ff]                  */
+  const float* final_norm; /* [d]        RMSNorm gain before the head */
+  const float* head_w1;    /* [d, d]     head, first layer          */
+  const float* head_b1;    /* [d]                                   */
+  const float* head_w2;    /* [2, d]     head, second layer         */
+  const float* head_b2;    /* [2]                                   */
+} fsx_paper_weights;
+
+/* A tick handle for the ten-token layout (Sec. 3.1). cfg as for fsx_create, except
+ * that n_action, n_frame and n_waypoints are fixed by the layout (5 queries, the
+ * state token + 4 visual tokens, 5 waypoints; the given values are ignored) and
+ * frame_dtype is the dtype of the visual tokens. The handle is an fsx_handle: use
+ * fsx_paper_tick for its ticks, fsx_get_status, fsx_set_kernel_timing,
+ * fsx_kernel_time and fsx_destroy as usual. Blocking. Errors as fsx_create. */
+fsx_status fsx_paper_create(const fsx_config* cfg, const fsx_paper_weights* w, int device, fsx_handle* out);
+
+/* One tick of the ten-token layout for B vehicles (Sec. 3.1, Eq. 1).
+ *   k_cache, v_cache, d_offsets : as fsx_tick.
+ *   d_visual    : DEVICE [B, 4, d] visual tokens of the current frame (cfg.frame_dtype).
+ *   d_state     : DEVICE fp32 [B, 16] ego state (order above).
+ *   d_waypoints : DEVICE fp32 [B, 5, 2] output.
+ * Enqueued on `stream`: the state MLP writes the frame rows into a handle-owned
+ * buffer, then the tick runs; device-side errors as fsx_tick (no waypoint written). */
+fsx_status fsx_paper_tick(fsx_handle h, const void* const* k_cache, const void* const* v_cache,
+                          const int64_t* d_offsets, int B, const void* d_visual, const float* d_state,
+                          float* d_waypoints, void* stream);
+
 /* ================================================================== cache append
  * The slow system's incremental forward (Sec. 1, Sec. 3.3): every K = 4 ticks
  * the current frame's n_new (4) tokens go through the frozen backbone -- a

@@ -113,6 +113,13 @@ struct fsx_handle_s {
   cudaStream_t last_stream = nullptr;
   bool has_last = false;
   std::mutex mu;
+  // the ten-token layout (paper_tokens.cu): two-layer head and state MLP parameters,
+  // assembled frame rows; null for the 42-token tick
+  float* paper_params = nullptr;
+  const float* paper_head = nullptr;
+  const float* paper_state_w = nullptr;
+  float* paper_frames = nullptr;
+  int paper_visual_dtype = 0;
 };
 
 namespace {
@@ -203,10 +210,24 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     pa.counters = h->p_counters;
     pa.status = h->status;
     pa.attn_capture = attn_capture;
+    pa.head = h->paper_head == nullptr ? 1 : 0;
     FSX_CUDA(cudaMemsetAsync(h->p_counters, 0, sizeof(int) * (2 * c.n_layers + 1), st));
     FSX_CUDA(mark(kClassPersistent, true));
     FSX_CUDA(fsx::launch_persistent(pa, c.cache_dtype, st));
     FSX_CUDA(mark(kClassPersistent, false));
+    if (h->paper_head != nullptr) {  // the two-layer head over the final residual buffer
+      fsx::Head2Args h2{};
+      h2.x = h->p_x + static_cast<size_t>((2 * c.n_layers) % 3) * fsx::kTokTile * d;
+      h2.vehicle_rows = 0;
+      h2.final_norm = h->final_norm;
+      h2.w = h->paper_head;
+      h2.targs = h->d_args;
+      h2.d = d;
+      h2.n_waypoints = c.n_waypoints;
+      h2.B = 1;
+      h2.status = h->status;
+      FSX_CUDA(fsx::launch_head2(h2, st, false));
+    }
     if (timed) h->timed_pairs = pair;
     return FSX_OK;
   }
@@ -352,7 +373,21 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
   ha.n_waypoints = c.n_waypoints;
   ha.B = B;
   ha.status = h->status;
-  FSX_CUDA(fsx::launch_head(ha, st, pdl));
+  if (h->paper_head != nullptr) {
+    fsx::Head2Args h2{};
+    h2.x = h->x;
+    h2.vehicle_rows = T;
+    h2.final_norm = h->final_norm;
+    h2.w = h->paper_head;
+    h2.targs = h->d_args;
+    h2.d = d;
+    h2.n_waypoints = c.n_waypoints;
+    h2.B = B;
+    h2.status = h->status;
+    FSX_CUDA(fsx::launch_head2(h2, st, pdl));
+  } else {
+    FSX_CUDA(fsx::launch_head(ha, st, pdl));
+  }
   if (timed) h->timed_pairs = pair;
   return FSX_OK;
 }
@@ -433,6 +468,8 @@ void free_handle(fsx_handle_s* h) {
   for (cudaEvent_t e : h->tev) cudaEventDestroy(e);
   if (h->last_tick) cudaEventDestroy(h->last_tick);
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
+  if (h->paper_params) cudaFree(h->paper_params);
+  if (h->paper_frames) cudaFree(h->paper_frames);
   void* bufs[] = {h->p_arena, h->p_x, h->p_counters, h->w_arena, h->params, h->x, h->x16, h->ss, h->qkv, h->o, h->hbuf, h->part,
                   h->gemm_part, h->tile_count, h->order, h->status, h->d_args,
                   h->st_offsets, h->st_frames, h->st_waypoints};
@@ -442,6 +479,33 @@ void free_handle(fsx_handle_s* h) {
 }
 
 }  // namespace
+
+namespace fsx {
+
+// hooks of the ten-token layout (paper_tokens.cu)
+fsx_status paper_attach(fsx_handle h, float* d_params, const float* d_head, float* d_frames, const float* d_state_w,
+                        int visual_dtype) {
+  h->paper_params = d_params;
+  h->paper_head = d_head;
+  h->paper_frames = d_frames;
+  h->paper_state_w = d_state_w;
+  h->paper_visual_dtype = visual_dtype;
+  return FSX_OK;
+}
+float* paper_frames(fsx_handle h) { return h->paper_frames; }
+const float* paper_state_weights(fsx_handle h) { return h->paper_state_w; }
+int paper_device(fsx_handle h) { return h->device; }
+int paper_max_batch(fsx_handle h) { return h->cfg.max_batch; }
+int paper_d(fsx_handle h) { return h->cfg.d_model; }
+int paper_visual_dtype(fsx_handle h) { return h->paper_visual_dtype; }
+// order work on `st` after the handle's previous tick when that ran on another stream
+cudaError_t paper_order_after_last_tick(fsx_handle h, cudaStream_t st) {
+  std::lock_guard<std::mutex> lock(h->mu);
+  if (h->has_last && h->last_stream != st) return cudaStreamWaitEvent(st, h->last_tick, 0);
+  return cudaSuccess;
+}
+
+}  // namespace fsx
 
 extern "C" {
 
@@ -792,7 +856,7 @@ long long fsx_weight_bytes(fsx_handle h) { return h ? h->weight_bytes : 0; }
 
 int fsx_tick_launches(fsx_handle h, int B) {
   if (!h || B < 1) return 0;
-  if (use_persistent(h, B)) return 1;
+  if (use_persistent(h, B)) return h->paper_head != nullptr ? 2 : 1;
   return 2 + h->cfg.n_layers * (4 + fsx::attention_launch_count(attention_splits(h, B)));
 }
 

@@ -96,6 +96,31 @@ struct HeadArgs {
 };
 cudaError_t launch_head(const HeadArgs& a, cudaStream_t stream, bool pdl);
 
+// Two-layer waypoint head of the ten-token layout (Sec. 3.1): waypoint j of vehicle b =
+// W_h2 silu(W_h1 RMSNorm(x_{b,j}; g_f) + b_h1) + b_h2, read from token row j of the vehicle.
+struct Head2Args {
+  const float* x;          // token row j of vehicle b at x + (b * vehicle_rows + j) * d
+  long long vehicle_rows;  // token rows per vehicle in x
+  const float* final_norm; // [d]
+  const float* w;          // W_h1 [d, d], b_h1 [d], W_h2 [2, d], b_h2 [2], fp32 row-major [out, in]
+  const TickArgs* targs;   // waypoint output pointer
+  int d, n_waypoints, B;
+  int* status;             // no waypoint is written when it is set
+};
+cudaError_t launch_head2(const Head2Args& a, cudaStream_t stream, bool pdl);
+
+// State token and visual tokens of the ten-token layout into a tick's fp32 frame rows:
+// frames[b, 0] = W_s2 silu(W_s1 state_b + b_s1) + b_s2, frames[b, 1 + i] = visual[b, i].
+struct StateArgs {
+  const float* state;      // [B, 16]
+  const void* visual;      // [B, 4, d] of visual_dtype (fsx_dtype)
+  int visual_dtype;
+  const float* w;          // W_s1 [d, 16], b_s1 [d], W_s2 [d, d], b_s2 [d]
+  float* frames;           // [B, 5, d]
+  int d, B;
+};
+cudaError_t launch_state_tokens(const StateArgs& a, cudaStream_t stream);
+
 // Launch helper: cudaLaunchKernelEx with the programmatic-stream-serialisation
 // attribute when `pdl` is set and a (cluster_x, cluster_y, 1) cluster when either exceeds 1.
 cudaError_t launch_ex(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t stream,

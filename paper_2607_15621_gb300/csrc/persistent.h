@@ -35,6 +35,7 @@ struct PersistArgs {
   int* counters;                // [2 n_layers + 1], zeroed before every launch
   int* status;
   __half* attn_capture;         // optional [n_layers][T][H*128]
+  int head;                     // 1: CTA 0 runs the single-layer waypoint head; 0: a later launch does
 };
 
 size_t persistent_smem_bytes(int d);

@@ -1135,7 +1135,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
 
   // =========================== head ===========================
-  if (cta == 0) {
+  if (cta == 0 && p.head) {
     wait_counter(p.counters + 2 * p.n_layers, n_b_ctas, p.status, abort);
     // a tick with a device-side error (an out-of-range cache value, a timeout) writes no waypoint
     if (*reinterpret_cast<volatile int*>(p.status) != 0) return;

@@ -53,6 +53,15 @@ class Weights(ctypes.Structure):
     _fields_ = [(name, ctypes.POINTER(ctypes.c_float)) for name in _WEIGHT_FIELDS]
 
 
+_PAPER_WEIGHT_FIELDS = ["state_w1", "state_b1", "state_w2", "state_b2", "query_emb", "pos_emb", "attn_norm", "wq",
+                        "wk", "wv", "wo", "mlp_norm", "w_gate", "w_up", "w_down", "final_norm", "head_w1", "head_b1",
+                        "head_w2", "head_b2"]
+
+
+class PaperWeights(ctypes.Structure):
+    _fields_ = [(name, ctypes.POINTER(ctypes.c_float)) for name in _PAPER_WEIGHT_FIELDS]
+
+
 class AppendConfig(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int), ("d_model", ctypes.c_int), ("n_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("d_ff", ctypes.c_int), ("n_new", ctypes.c_int),
@@ -93,6 +102,8 @@ def _load():
         "fsx_attention_noalloc": (i32, [vp, ctypes.c_longlong, vp, vp, ctypes.c_longlong, i32, i32, vp, vp,
                                         i32, vp, i32, i32, i32, i32, vp, vp, vp]),
         "fsx_attention_noalloc_status": (i32, [vp]),
+        "fsx_paper_create": (i32, [ctypes.POINTER(Config), ctypes.POINTER(PaperWeights), i32, ctypes.POINTER(vp)]),
+        "fsx_paper_tick": (i32, [vp, vpp, vpp, vp, i32, vp, vp, vp, vp]),
         "fsx_append_create": (i32, [ctypes.POINTER(AppendConfig), ctypes.POINTER(AppendWeights), i32,
                                     ctypes.POINTER(vp)]),
         "fsx_append": (i32, [vp, vpp, vpp, vp, vp, i32, vp, vp, vp]),
@@ -122,7 +133,7 @@ def declared_symbols() -> list[str]:
             "fsx_get_status", "fsx_last_error",
             "fsx_destroy", "fsx_weight_bytes", "fsx_tick_launches", "fsx_set_kernel_timing",
             "fsx_kernel_time", "fsx_attention_workspace_bytes", "fsx_attention", "fsx_attention_noalloc",
-            "fsx_attention_noalloc_status", "fsx_append_create", "fsx_append", "fsx_append_get_status", "fsx_append_weight_bytes",
+            "fsx_attention_noalloc_status", "fsx_paper_create", "fsx_paper_tick", "fsx_append_create", "fsx_append", "fsx_append_get_status", "fsx_append_weight_bytes",
             "fsx_append_destroy"]
 
 
@@ -245,6 +256,29 @@ class Expert:
         n = ctypes.c_int()
         check(lib().fsx_kernel_time(self.h, ctypes.byref(ms), ctypes.byref(n)))
         return float(ms.value), int(n.value)
+
+
+class PaperExpert(Expert):
+    """A tick handle of the paper's ten-token layout (fsx_paper_create / fsx_paper_tick):
+    state token, four visual tokens, five waypoint queries and a two-layer head over the
+    same layer stack. Argument marshalling only."""
+
+    def __init__(self, dims: Dims, weights: dict, max_batch: int, max_total_cache_tokens: int,
+                 cache_dtype: str = "bf16", visual_dtype: str = "bf16", device: int = 0):
+        self.dims = dims
+        self.cfg = make_config(dims, max_batch, max_total_cache_tokens, cache_dtype, visual_dtype)
+        keep = {k: np.ascontiguousarray(weights[k], dtype=np.float32) for k in _PAPER_WEIGHT_FIELDS}
+        wst = PaperWeights(*[keep[k].ctypes.data_as(ctypes.POINTER(ctypes.c_float)) for k in _PAPER_WEIGHT_FIELDS])
+        h = ctypes.c_void_p()
+        check(lib().fsx_paper_create(ctypes.byref(self.cfg), ctypes.byref(wst), device, ctypes.byref(h)))
+        self.h = h
+        del keep
+
+    def paper_tick(self, k_layers, v_layers, offsets, visual, state, out, stream=None):
+        B = int(visual.shape[0])
+        check(lib().fsx_paper_tick(self.h, _ptr_array(k_layers), _ptr_array(v_layers), _ptr(offsets), B,
+                                   _ptr(visual), _ptr(state), _ptr(out), _stream(stream)))
+        return out
 
 
 def attention_workspace_bytes(B: int, n_heads: int, n_q: int, n_splits: int) -> int:

@@ -93,6 +93,11 @@ APPEND_WORKLOADS = {
     "append_b1_l224": dict(batch=1, length=224),
 }
 
+# The paper's ten-token layout (Sec. 3.1): `batch` vehicles, each with `length` cached tokens.
+PAPER_WORKLOADS = {
+    "paper_b1_l224": dict(batch=1, length=224),
+}
+
 # Workloads: name -> (batch, length spec, dtype). Length spec is either a fixed
 # per-vehicle cache length or a (lo, hi) inclusive uniform range.
 WORKLOADS = {
@@ -112,6 +117,8 @@ _STREAM_FRAMES = 0x5EED0003
 _STREAM_LENGTHS = 0x5EED0004
 _STREAM_BACKBONE = 0x5EED0005
 _STREAM_APPEND_TOKENS = 0x5EED0006
+_STREAM_PAPER_WEIGHTS = 0x5EED0007
+_STREAM_PAPER_INPUTS = 0x5EED0008
 
 
 def _gen(seed: int, stream: int, device="cpu") -> torch.Generator:
@@ -234,3 +241,47 @@ def make_append_tokens(dims: BackboneDims, batch: int, seed: int = 0, device="cp
     g = _gen(seed, _STREAM_APPEND_TOKENS, device=dev.type if dev.type == "cpu" else dev)
     x = torch.randn(batch, dims.n_new, dims.d_model, generator=g, device=dev)
     return x.to(torch.bfloat16).contiguous()
+
+
+PAPER_STATE_DIM = 16
+PAPER_VISUAL = 4
+PAPER_QUERIES = 5
+
+
+def make_paper_weights(dims: Dims = EXPERT, seed: int = 0, dtype: str = "fp32") -> dict:
+    """Weights of the paper's ten-token layout: the layer stack of make_weights (same seed)
+    plus the state MLP (W_s1 ~ N(0, 1/16), W_s2 ~ N(0, 1/d), biases ~ N(0, 0.1^2)), the
+    five waypoint queries and the [10, d] position table (~ N(0, 0.02^2)), and the
+    two-layer head (W_h1 ~ N(0, 1/d), W_h2 ~ N(0, 1/d), biases ~ N(0, 0.1^2))."""
+    base = make_weights(dims, seed, dtype)
+    g = _gen(seed, _STREAM_PAPER_WEIGHTS)
+    d = dims.d_model
+
+    def normal(shape, std):
+        return torch.randn(*shape, generator=g, dtype=torch.float32) * std
+
+    extra = {
+        "state_w1": normal((d, PAPER_STATE_DIM), 1.0 / math.sqrt(PAPER_STATE_DIM)),
+        "state_b1": normal((d,), 0.1),
+        "state_w2": normal((d, d), 1.0 / math.sqrt(d)),
+        "state_b2": normal((d,), 0.1),
+        "query_emb": normal((PAPER_QUERIES, d), 0.02),
+        "pos_emb": normal((1 + PAPER_VISUAL + PAPER_QUERIES, d), 0.02),
+        "head_w1": normal((d, d), 1.0 / math.sqrt(d)),
+        "head_b1": normal((d,), 0.1),
+        "head_w2": normal((2, d), 1.0 / math.sqrt(d)),
+        "head_b2": normal((2,), 0.1),
+    }
+    w = {k: v for k, v in base.items() if k not in ("act_emb", "pos_emb", "head_w", "head_b")}
+    w.update({k: np.ascontiguousarray(_round(v, dtype).numpy()) for k, v in extra.items()})
+    return w
+
+
+def make_paper_inputs(dims: Dims, batch: int, seed: int = 0, dtype: str = "bf16", device="cpu"):
+    """Visual tokens [B, 4, d] (bfloat16 for "bf16", float32 for "fp32") ~ N(0, 1) and the
+    fp32 ego state [B, 16] ~ N(0, 1) of the ten-token layout."""
+    dev = torch.device(device)
+    g = _gen(seed, _STREAM_PAPER_INPUTS, device=dev.type if dev.type == "cpu" else dev)
+    visual = torch.randn(batch, PAPER_VISUAL, dims.d_model, generator=g, device=dev)
+    state = torch.randn(batch, PAPER_STATE_DIM, generator=g, device=dev)
+    return visual.to(torch.bfloat16 if dtype == "bf16" else torch.float32).contiguous(), state.contiguous()

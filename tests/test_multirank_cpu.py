@@ -120,3 +120,16 @@ def test_cpu_baseline_sample_spans_the_length_order():
     assert len(picks) == 8 and len(set(picks)) == 8
     assert int(np.argmin(lengths)) in picks and int(np.argmax(lengths)) in picks
     assert bench.baseline_vehicles([224]) == [0]
+
+
+def test_paper_layout_reference_arm_prints_one_line():
+    """The ten-token workload's reference arm: its fp64 oracle (one expert layer here)."""
+    cmd = [sys.executable, "bench.py", "--impl", "reference", "--workload", "paper_b1_l224", "--layers", "1",
+           "--steps", "1", "--warmup", "1", "--cpu-seconds", "1"]
+    res = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600)
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [l for l in res.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, res.stdout
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["value"] > 0
+    assert line["config"]["workload"] == "paper_b1_l224" and line["config"]["tokens_per_vehicle"] == 10

@@ -111,3 +111,30 @@ def test_clip_prefixes_follow_the_visibility_rule():
     want = [staleness_oracle.visible_prefix(j, c["delta"], c["text"], c["tokens_per_frame"]) for j in range(c["frames"])]
     assert list(got) == want
     assert got.max() <= c["text"] + c["tokens_per_frame"] * c["frames"]
+
+
+def test_paper_layout_recipe():
+    """Ten-token layout inputs: the layer stack of make_weights plus the state MLP, queries,
+    positions and the two-layer head with the stated scales; ego state and visual tokens
+    N(0, 1)."""
+    import math
+    from paper_2607_15621_gb300 import synth
+    dims = synth.Dims(n_layers=2, n_action=5, n_frame=5)
+    w = synth.make_paper_weights(dims, 0, "fp32")
+    base = synth.make_weights(dims, 0, "fp32")
+    assert np.array_equal(w["wq"], base["wq"]) and np.array_equal(w["final_norm"], base["final_norm"])
+    d = dims.d_model
+    shapes = {"state_w1": (d, 16), "state_w2": (d, d), "query_emb": (5, d), "pos_emb": (10, d), "head_w1": (d, d),
+              "head_w2": (2, d), "head_b2": (2,)}
+    for k, shp in shapes.items():
+        assert w[k].shape == shp, k
+    assert abs(w["state_w1"].std() - 1 / 4) < 0.02
+    assert abs(w["state_w2"].std() - 1 / math.sqrt(d)) < 0.003
+    assert abs(w["head_w1"].std() - 1 / math.sqrt(d)) < 0.003
+    assert abs(w["query_emb"].std() - 0.02) < 0.002 and abs(w["pos_emb"].std() - 0.02) < 0.002
+    assert "act_emb" not in w and "head_w" not in w
+    visual, state = synth.make_paper_inputs(dims, 3, 0, "bf16")
+    assert visual.shape == (3, 4, d) and visual.dtype == torch.bfloat16 and state.shape == (3, 16)
+    assert abs(float(visual.float().std()) - 1.0) < 0.05
+    v2, s2 = synth.make_paper_inputs(dims, 3, 0, "bf16")
+    assert torch.equal(visual, v2) and torch.equal(state, s2)
