@@ -18,6 +18,9 @@ exceed the 129 MB L2, so no flush is needed between ticks.
 The workload `clip_j40_delta1` times the staleness-masked forward over a 40-frame
 clip (Sec. 3.2: every frame block over the cache prefix ending one frame earlier,
 all blocks in one tick over explicit row ranges); value = frame-blocks/s.
+The workload `fastslow_b1_l224` paces one vehicle's ticks (every 12.5 ms) with a cache
+append before every 4th tick through an fsx session (Sec. 3.3) and reports the tick
+latency distribution in the serial and the concurrent schedule.
 The workload `paper_b1_l224` times the paper's own ten-token layout (state token,
 four visual tokens, five queries, two-layer head; Sec. 3.1) at B = 1, L = 224.
 The workload `append_b1_l224` instead times the backbone's incremental cache
@@ -727,6 +730,111 @@ def run_paper(args):
         dist.destroy_process_group()
 
 
+FASTSLOW_METRIC = "vehicle-ticks/s (1e6 / mean tick latency) of the expert tick while the cache append runs every 4 ticks"
+
+
+def run_fastslow_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    print(json.dumps({"impl": "reference", "unavailable": "the fast-slow schedule is a GPU stream schedule; its "
+                      "arithmetic (the tick and the append) has reference arms of its own "
+                      "(--workload bf16_b1_l224, --workload append_b1_l224)"}))
+
+
+def run_fastslow(args):
+    """Ticks of one vehicle paced at a fixed cadence with a 4-token cache append issued
+    before every k-th tick, through an fsx session, in the serial and the concurrent
+    schedule. A tick's latency runs from its issue (an event on an idle stream) to the end
+    of its work on the tick stream, so it includes any wait for, or contention with, an
+    append."""
+    import torch
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2607_15621_gb300 import fsx, synth
+    spec = synth.FASTSLOW_WORKLOADS[args.workload]
+    dims = synth.EXPERT if args.layers is None else dataclasses.replace(synth.EXPERT, n_layers=args.layers)
+    bdims = dataclasses.replace(synth.BACKBONE, n_layers=dims.n_layers)
+    L0, K, cadence = spec["length"], spec["k"], spec["cadence_ms"] / 1e3
+    n_ticks = args.steps
+    cap = L0 + (n_ticks // K + 8) * bdims.n_new + 64
+    w = synth.make_weights(dims, 0, "bf16")
+    bw = synth.make_backbone_weights(bdims, 0, "bf16")
+    k0, v0, _ = synth.make_cache(dims, [L0], 0, "bf16", device=dev)
+    frames = synth.make_frames(dims, 1, 0, "bf16", device=dev)
+    x = synth.make_append_tokens(bdims, 1, 0, device=dev)
+    hidden = torch.empty(1, bdims.n_new, bdims.d_model, device=dev)
+    out = torch.empty(1, dims.n_waypoints, 2, device=dev)
+    ex = fsx.Expert(dims, w, 1, cap, device=local)
+    ap = fsx.Append(bdims, bw, 1, cap, device=local)
+    del w, bw
+    clock = torch.cuda.Stream(dev)
+    modes = {}
+    for name, concurrent in (("serial", False), ("concurrent", True)):
+        kc = [torch.zeros(cap, dims.n_heads, dims.head_dim, dtype=torch.bfloat16, device=dev) for _ in k0]
+        vc = [torch.zeros_like(t) for t in kc]
+        for dst, src in zip(kc + vc, k0 + v0):
+            dst[:L0] = src
+        ses = fsx.Session(ex, ap, kc, vc, cap, L0, concurrent, device=local)
+        tick_stream = torch.cuda.ExternalStream(ses.tick_stream(), device=dev)
+        app_stream = torch.cuda.ExternalStream(ses.append_stream(), device=dev)
+        for i in range(8):  # warm-up, appends included
+            if i % K == 0:
+                ses.append(x, hidden)
+            ses.tick(frames, out)
+        ses.sync()
+        pairs, apairs, snaps = [], [], []
+        t0 = time.perf_counter()
+        for i in range(n_ticks):
+            wait = t0 + i * cadence - time.perf_counter()
+            if wait > 0:
+                time.sleep(wait)
+            if i % K == 0:
+                a0 = torch.cuda.Event(enable_timing=True)
+                a1 = torch.cuda.Event(enable_timing=True)
+                a0.record(app_stream)
+                ses.append(x, hidden)
+                a1.record(app_stream)
+                apairs.append((a0, a1))
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(clock)
+            snaps.append(ses.tick(frames, out))
+            e1.record(tick_stream)
+            pairs.append((e0, e1))
+        ses.sync()
+        if ex.status() != fsx.FSX_OK or ap.status() != fsx.FSX_OK:
+            raise RuntimeError("device status set during the fast-slow schedule")
+        lat = np.array([a.elapsed_time(b) * 1e3 for a, b in pairs])
+        app = np.array([a.elapsed_time(b) * 1e3 for a, b in apairs])
+        modes[name] = {"ticks": n_ticks, "tick_latency_us": {
+                           "p50": float(np.percentile(lat, 50)), "p90": float(np.percentile(lat, 90)),
+                           "p99": float(np.percentile(lat, 99)), "max": float(lat.max()), "mean": float(lat.mean()),
+                           "with_append_issued_p50": float(np.percentile(lat[::K], 50)),
+                           "without_append_p50": float(np.percentile(np.delete(lat, np.s_[::K]), 50))},
+                       "append_us": {"p50": float(np.percentile(app, 50)), "max": float(app.max())},
+                       "snapshot_rows": {"first": int(snaps[0]), "last": int(snaps[-1]),
+                                         "stale_ticks": int(sum(1 for i, s_ in enumerate(snaps)
+                                                                if i % K == 0 and s_ < snaps[min(i + 1, n_ticks - 1)]))}}
+        ses.close()
+        del kc, vc
+    ex.close()
+    ap.close()
+    conc = modes["concurrent"]["tick_latency_us"]
+    line = {
+        "metric": FASTSLOW_METRIC, "value": 1e6 / conc["mean"], "unit": UNIT, "n_gpus": 1, "steps": n_ticks,
+        "warmup": 8, "ms_per_step": conc["mean"] / 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f16 (fp32 accumulate)",
+        "data": "synthetic (seeded N(0,1) cache/frames/new tokens, N(0,1/fan_in) weights)",
+        "config": {"workload": args.workload, "cache_len": L0, "append_every": K, "cadence_ms": spec["cadence_ms"],
+                   "layers": dims.n_layers, "backbone_d_model": bdims.d_model, "new_tokens": bdims.n_new},
+        "gpu_launches": None, "schedules": modes,
+    }
+    if rank == 0:
+        print(json.dumps(line))
+
+
 def run_reference(args):
     world, rank, _ = dist_env()
     if rank != 0:
@@ -827,6 +935,9 @@ def main():
         return
     if args.workload in synth.CLIP_WORKLOADS:
         (run_clip_reference if args.impl == "reference" else run_clip)(args)
+        return
+    if args.workload in synth.FASTSLOW_WORKLOADS:
+        (run_fastslow_reference if args.impl == "reference" else run_fastslow)(args)
         return
     if args.workload in synth.PAPER_WORKLOADS:
         (run_paper_reference if args.impl == "reference" else run_paper)(args)

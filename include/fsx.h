@@ -389,11 +389,66 @@ fsx_status fsx_append(fsx_append_handle h, void* const* k_cache, void* const* v_
  * word (FSX_OK or FSX_ERR_DEVICE_ARG). */
 fsx_status fsx_append_get_status(fsx_append_handle h, void* stream);
 
+/* enable = 1: later appends on this handle run no kernel that waits on other CTAs
+ * (the residual GEMMs are not split along K), so an append can share the GPU with a
+ * tick whose single-launch kernel needs all of its CTAs resident (the concurrent
+ * schedule of fsx_session). Slower per append; enable = 0 restores the default. */
+fsx_status fsx_append_set_concurrent(fsx_append_handle h, int enable);
+
 /* Bytes of the handle's fp16 weight arena (algorithmic weight bytes per call). */
 long long fsx_append_weight_bytes(fsx_append_handle h);
 
 /* Releases the handle's device memory (synchronises its device). */
 void fsx_append_destroy(fsx_append_handle h);
+
+/* ====================================================== the asynchronous fast-slow schedule
+ * Sec. 3.3 and Fig. 1: the fast system ticks every 50 ms on the cache as it stands,
+ * while every K = 4 ticks the slow system appends the newest frame's tokens behind
+ * it. A session drives one vehicle's tick handle and append handle over one cache:
+ * it owns the cache's committed length, gives every append the rows after everything
+ * already reserved, and gives every tick a snapshot -- the rows of the appends that
+ * have completed -- so a tick never reads a row that is being written and the
+ * append-only cache needs no lock.
+ *   FSX_SCHED_SERIAL     appends run on the tick stream: a tick waits for an append
+ *                        in flight and reads its rows.
+ *   FSX_SCHED_CONCURRENT appends run on a low-priority stream of their own, ticks on
+ *                        a high-priority stream; the append handle is switched to
+ *                        fsx_append_set_concurrent(h, 1), so no append kernel waits
+ *                        on other CTAs and the single-launch tick always gets its SMs.
+ * The session never frees the handles or the cache; destroy it before them. */
+typedef struct fsx_session_s* fsx_session;
+enum { FSX_SCHED_SERIAL = 0, FSX_SCHED_CONCURRENT = 1 };
+
+/* tick: an fsx_handle whose max_total_cache_tokens >= capacity_rows (one vehicle);
+ * append: an fsx_append_handle with the same n_layers and n_new tokens per call and
+ * max_cache_rows >= capacity_rows; k_cache, v_cache: HOST arrays of n_layers DEVICE
+ * pointers to bf16 [capacity_rows, n_heads, head_dim] buffers whose first
+ * committed_rows rows hold the cache. Creates the session's two streams. */
+fsx_status fsx_session_create(fsx_handle tick, fsx_append_handle append, void* const* k_cache, void* const* v_cache,
+                              int n_layers, int n_new, long long capacity_rows, long long committed_rows, int mode,
+                              int device, fsx_session* out);
+
+/* Enqueue one append of n_new tokens (d_x_new: DEVICE bf16 [1, n_new, d_backbone])
+ * at the rows after everything reserved so far, attending to all of them; the hidden
+ * states go to d_hidden (DEVICE fp32 [1, n_new, d_backbone]). Asynchronous on the
+ * session's append stream. FSX_ERR_INVALID_ARG when the rows would pass the capacity. */
+fsx_status fsx_session_append(fsx_session s, const void* d_x_new, float* d_hidden);
+
+/* Enqueue one tick (d_frames: DEVICE [1, n_frame, d] of the tick handle's frame dtype)
+ * over the current snapshot on the session's tick stream; *snapshot_rows (if not NULL)
+ * receives the number of cache rows the tick reads. */
+fsx_status fsx_session_tick(fsx_session s, const void* d_frames, float* d_waypoints, long long* snapshot_rows);
+
+/* Rows of completed appends (retires finished appends; does not block), and rows
+ * reserved including appends in flight. */
+long long fsx_session_committed(fsx_session s);
+long long fsx_session_reserved(fsx_session s);
+/* The session's tick and append streams (cudaStream_t), e.g. to time them. */
+void* fsx_session_tick_stream(fsx_session s);
+void* fsx_session_append_stream(fsx_session s);
+/* Waits for every append and tick enqueued so far. */
+fsx_status fsx_session_sync(fsx_session s);
+void fsx_session_destroy(fsx_session s);
 
 #ifdef __cplusplus
 }

@@ -21,7 +21,7 @@ OUT_DIR = os.path.join(PKG, "_lib")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libfsx.so")
 SOURCES = ["fsx.cu", "launch.cu", "gemm_tc.cu", "attention.cu", "attention_tc.cu", "embed_head.cu",
-           "attention_noalloc.cu", "tick_persistent.cu", "append.cu", "paper_tokens.cu"]
+           "attention_noalloc.cu", "tick_persistent.cu", "append.cu", "paper_tokens.cu", "session.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-pthread",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]

@@ -283,6 +283,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32) append_attn_kernel(const Attn
 struct fsx_append_s {
   fsx_append_config cfg{};
   int device = 0;
+  bool concurrent = false;  // no kernel of a call waits on other CTAs (no split K)
   int sm_count = 0;
   int HD = 0;
   void* w_arena = nullptr;
@@ -470,6 +471,12 @@ fsx_status fsx_append_create(const fsx_append_config* cfg, const fsx_append_weig
   return FSX_OK;
 }
 
+fsx_status fsx_append_set_concurrent(fsx_append_handle h, int enable) {
+  if (!h) return fail(FSX_ERR_INVALID_ARG, "handle is NULL");
+  h->concurrent = enable != 0;
+  return FSX_OK;
+}
+
 fsx_status fsx_append(fsx_append_handle h, void* const* k_cache, void* const* v_cache, const int64_t* d_offsets,
                       const int64_t* d_dst_rows, int B, const void* d_x_new, float* d_hidden, void* stream) {
   if (!h) return fail(FSX_ERR_INVALID_ARG, "handle is NULL");
@@ -558,7 +565,7 @@ fsx_status fsx_append(fsx_append_handle h, void* const* k_cache, void* const* v_
     go.ldxo = d;
     go.ss_out = h->ss;
     go.ss_stride = h->ss_stride;
-    go.k_splits = fsx::gemm_tc_k_splits((d / 128) * m_tiles, HD / 64, h->sm_count);
+    go.k_splits = h->concurrent ? 1 : fsx::gemm_tc_k_splits((d / 128) * m_tiles, HD / 64, h->sm_count);
     go.part = h->gemm_part;
     go.tile_count = h->tile_count;
     FSX_CUDA(fsx::launch_gemm_tc(h->map_o[bn_i], go, bn, fsx::kEpiResidual, false, st, false));
@@ -587,7 +594,7 @@ fsx_status fsx_append(fsx_append_handle h, void* const* k_cache, void* const* v_
     gd.ldxo = d;
     gd.ss_out = h->ss;
     gd.ss_stride = h->ss_stride;
-    gd.k_splits = fsx::gemm_tc_k_splits((d / 128) * m_tiles, F / 64, h->sm_count);
+    gd.k_splits = h->concurrent ? 1 : fsx::gemm_tc_k_splits((d / 128) * m_tiles, F / 64, h->sm_count);
     gd.part = h->gemm_part;
     gd.tile_count = h->tile_count;
     FSX_CUDA(fsx::launch_gemm_tc(h->map_h[bn_i], gd, bn, fsx::kEpiResidual, false, st, false));

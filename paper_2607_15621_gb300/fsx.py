@@ -27,6 +27,8 @@ FSX_ERR_DEVICE_ARG = 6
 FSX_ERR_RANGE = 7
 FSX_F32 = 0
 FSX_BF16 = 1
+FSX_SCHED_SERIAL = 0
+FSX_SCHED_CONCURRENT = 1
 
 KCLASS = {"qkv": 0, "attention": 1, "out_proj": 2, "gate_up": 3, "down": 4, "persistent": 5}
 
@@ -104,6 +106,17 @@ def _load():
         "fsx_attention_noalloc_status": (i32, [vp]),
         "fsx_paper_create": (i32, [ctypes.POINTER(Config), ctypes.POINTER(PaperWeights), i32, ctypes.POINTER(vp)]),
         "fsx_paper_tick": (i32, [vp, vpp, vpp, vp, i32, vp, vp, vp, vp]),
+        "fsx_append_set_concurrent": (i32, [vp, i32]),
+        "fsx_session_create": (i32, [vp, vp, vpp, vpp, i32, i32, ctypes.c_longlong, ctypes.c_longlong, i32, i32,
+                                     ctypes.POINTER(vp)]),
+        "fsx_session_append": (i32, [vp, vp, vp]),
+        "fsx_session_tick": (i32, [vp, vp, vp, ctypes.POINTER(ctypes.c_longlong)]),
+        "fsx_session_committed": (ctypes.c_longlong, [vp]),
+        "fsx_session_reserved": (ctypes.c_longlong, [vp]),
+        "fsx_session_tick_stream": (vp, [vp]),
+        "fsx_session_append_stream": (vp, [vp]),
+        "fsx_session_sync": (i32, [vp]),
+        "fsx_session_destroy": (None, [vp]),
         "fsx_append_create": (i32, [ctypes.POINTER(AppendConfig), ctypes.POINTER(AppendWeights), i32,
                                     ctypes.POINTER(vp)]),
         "fsx_append": (i32, [vp, vpp, vpp, vp, vp, i32, vp, vp, vp]),
@@ -133,8 +146,11 @@ def declared_symbols() -> list[str]:
             "fsx_get_status", "fsx_last_error",
             "fsx_destroy", "fsx_weight_bytes", "fsx_tick_launches", "fsx_set_kernel_timing",
             "fsx_kernel_time", "fsx_attention_workspace_bytes", "fsx_attention", "fsx_attention_noalloc",
-            "fsx_attention_noalloc_status", "fsx_paper_create", "fsx_paper_tick", "fsx_append_create", "fsx_append", "fsx_append_get_status", "fsx_append_weight_bytes",
-            "fsx_append_destroy"]
+            "fsx_attention_noalloc_status", "fsx_paper_create", "fsx_paper_tick", "fsx_append_create", "fsx_append",
+            "fsx_append_get_status", "fsx_append_weight_bytes", "fsx_append_destroy", "fsx_append_set_concurrent",
+            "fsx_session_create", "fsx_session_append", "fsx_session_tick", "fsx_session_committed",
+            "fsx_session_reserved", "fsx_session_tick_stream", "fsx_session_append_stream", "fsx_session_sync",
+            "fsx_session_destroy"]
 
 
 def last_error() -> str:
@@ -350,3 +366,52 @@ class Append:
 
     def weight_bytes(self) -> int:
         return int(lib().fsx_append_weight_bytes(self.h))
+
+
+class Session:
+    """An fsx_session: the asynchronous fast-slow schedule of one vehicle over one cache
+    (ticks on a snapshot of the committed rows, appends behind them). Marshalling only."""
+
+    def __init__(self, expert: "Expert", append: "Append", k_layers, v_layers, capacity_rows: int,
+                 committed_rows: int, concurrent: bool, device: int = 0):
+        self._keep = (list(k_layers), list(v_layers))
+        h = ctypes.c_void_p()
+        check(lib().fsx_session_create(expert.h, append.h, _ptr_array(k_layers), _ptr_array(v_layers),
+                                       len(k_layers), append.dims.n_new, capacity_rows, committed_rows,
+                                       FSX_SCHED_CONCURRENT if concurrent else FSX_SCHED_SERIAL, device,
+                                       ctypes.byref(h)))
+        self.h = h
+
+    def close(self):
+        if getattr(self, "h", None) and self.h.value:
+            lib().fsx_session_destroy(self.h)
+            self.h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def append(self, x_new, hidden):
+        check(lib().fsx_session_append(self.h, _ptr(x_new), _ptr(hidden)))
+
+    def tick(self, frames, out) -> int:
+        snap = ctypes.c_longlong()
+        check(lib().fsx_session_tick(self.h, _ptr(frames), _ptr(out), ctypes.byref(snap)))
+        return int(snap.value)
+
+    def committed(self) -> int:
+        return int(lib().fsx_session_committed(self.h))
+
+    def reserved(self) -> int:
+        return int(lib().fsx_session_reserved(self.h))
+
+    def tick_stream(self) -> int:
+        return lib().fsx_session_tick_stream(self.h)
+
+    def append_stream(self) -> int:
+        return lib().fsx_session_append_stream(self.h)
+
+    def sync(self):
+        check(lib().fsx_session_sync(self.h))

@@ -93,6 +93,12 @@ APPEND_WORKLOADS = {
     "append_b1_l224": dict(batch=1, length=224),
 }
 
+# The asynchronous fast-slow schedule (Sec. 3.3): one vehicle with `length` cached tokens,
+# a tick every `cadence_ms` and an append of 4 tokens before every `k`-th tick.
+FASTSLOW_WORKLOADS = {
+    "fastslow_b1_l224": dict(length=224, k=4, cadence_ms=12.5),
+}
+
 # The paper's ten-token layout (Sec. 3.1): `batch` vehicles, each with `length` cached tokens.
 PAPER_WORKLOADS = {
     "paper_b1_l224": dict(batch=1, length=224),
