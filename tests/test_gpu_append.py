@@ -148,3 +148,37 @@ def test_append_host_argument_errors():
             ap.append(kc, kc, off, None, x[:1], hidden)
     finally:
         ap.close()
+
+
+@pytest.mark.parametrize("concurrent", [False, True])
+def test_append_full_depth_one_vehicle(concurrent):
+    """All 32 layers of the backbone, one vehicle with the paper-shaped 224 cached tokens
+    (64 instruction + 40 frames x 4): the depth the bench runs, where bf16 rounding of the
+    written rows compounds over the layers. Both GEMM schedules (split K, and the one of the
+    concurrent fast-slow session without it)."""
+    dims = synth.BackboneDims()
+    w = synth.make_backbone_weights(dims, 1, "bf16")
+    L, n = 224, dims.n_new
+    k0, v0, _ = synth.make_cache(synth.Dims(n_layers=dims.n_layers), [L], 1, "bf16")
+    rows = L + n
+    kc = [torch.zeros(rows, H, D, dtype=torch.bfloat16, device="cuda") for _ in range(dims.n_layers)]
+    vc = [torch.zeros(rows, H, D, dtype=torch.bfloat16, device="cuda") for _ in range(dims.n_layers)]
+    for dst_t, src in zip(kc + vc, k0 + v0):
+        dst_t[:L] = src.cuda()
+    x = synth.make_append_tokens(dims, 1, seed=2).cuda()
+    ap = fsx.Append(dims, w, max_batch=1, max_cache_rows=rows)
+    try:
+        fsx.lib().fsx_append_set_concurrent(ap.h, 1 if concurrent else 0)
+        hidden = torch.empty(1, n, dims.d_model, device="cuda")
+        ap.append(kc, vc, torch.tensor([0, L], device="cuda"), torch.tensor([L], device="cuda"), x, hidden)
+        torch.cuda.synchronize()
+        assert ap.status() == fsx.FSX_OK
+        hidden = hidden.cpu().numpy()
+    finally:
+        ap.close()
+    h_ref, k_ref, v_ref = append_oracle.backbone_append(w, [t.float().numpy() for t in k0], [t.float().numpy() for t in v0],
+                                                        np.array([0, L]), x.float().cpu().numpy(), H, D)
+    assert row_err(hidden, h_ref).max() <= ROW_TOL
+    for l in range(dims.n_layers):
+        assert row_err(kc[l][L:].float().cpu().numpy(), k_ref[l]).max() <= ROW_TOL, l
+        assert row_err(vc[l][L:].float().cpu().numpy(), v_ref[l]).max() <= ROW_TOL, l
