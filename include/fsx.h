@@ -165,6 +165,14 @@ fsx_status fsx_tick_ranges_debug(fsx_handle h, const void* const* k_cache, const
  * error of those ticks; the tick that raised it wrote no waypoint). */
 fsx_status fsx_get_status(fsx_handle h, void* stream);
 
+/* For tests of the timeout path: the limit, in nanoseconds of the GPU's global timer,
+ * of the single-launch tick's device-wide waits (B = 1), 1 s by default (limit_ns = 0
+ * restores it). Not a passage of the paper. With a tiny limit a wait that finds its
+ * counter incomplete gives up at once: the tick ends with FSX_ERR_TIMEOUT and writes no
+ * waypoint, after letting everything it has in flight complete. Later ticks capture
+ * their graphs again with the new limit. Must not be called while ticks run. */
+fsx_status fsx_set_wait_limit(fsx_handle h, unsigned long long limit_ns);
+
 /* Thread-local message describing the last failure on this thread ("" if none). */
 const char* fsx_last_error(void);
 

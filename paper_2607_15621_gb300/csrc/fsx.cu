@@ -113,6 +113,7 @@ struct fsx_handle_s {
   cudaStream_t last_stream = nullptr;
   bool has_last = false;
   std::mutex mu;
+  unsigned long long wait_limit_ns = 1000000000ull;  // device-wide counter waits of the single-launch tick
   // the ten-token layout (paper_tokens.cu): two-layer head and state MLP parameters,
   // assembled frame rows; null for the 42-token tick
   float* paper_params = nullptr;
@@ -211,6 +212,7 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     pa.status = h->status;
     pa.attn_capture = attn_capture;
     pa.head = h->paper_head == nullptr ? 1 : 0;
+    pa.wait_limit_ns = h->wait_limit_ns;
     FSX_CUDA(cudaMemsetAsync(h->p_counters, 0, sizeof(int) * (2 * c.n_layers + 1), st));
     FSX_CUDA(mark(kClassPersistent, true));
     FSX_CUDA(fsx::launch_persistent(pa, c.cache_dtype, st));
@@ -851,6 +853,18 @@ fsx_status fsx_get_status(fsx_handle h, void* stream) {
 }
 
 void fsx_destroy(fsx_handle h) { free_handle(h); }
+
+fsx_status fsx_set_wait_limit(fsx_handle h, unsigned long long limit_ns) {
+  if (!h) return fail(FSX_ERR_INVALID_ARG, "handle is NULL");
+  std::lock_guard<std::mutex> lock(h->mu);
+  h->wait_limit_ns = limit_ns == 0 ? 1000000000ull : limit_ns;
+  // the graphs hold the limit as a kernel argument: capture them again
+  for (auto& kv : h->graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : h->timed_graphs) cudaGraphExecDestroy(kv.second);
+  h->graphs.clear();
+  h->timed_graphs.clear();
+  return FSX_OK;
+}
 
 long long fsx_weight_bytes(fsx_handle h) { return h ? h->weight_bytes : 0; }
 

@@ -36,6 +36,7 @@ struct PersistArgs {
   int* status;
   __half* attn_capture;         // optional [n_layers][T][H*128]
   int head;                     // 1: CTA 0 runs the single-layer waypoint head; 0: a later launch does
+  unsigned long long wait_limit_ns;  // limit of the device-wide counter waits (1 s unless a test lowers it)
 };
 
 size_t persistent_smem_bytes(int d);

@@ -79,7 +79,6 @@ constexpr int kNAcc = 4;                      // accumulators: one per MMA-issui
 constexpr uint32_t kAccCols = 64;             // tensor-memory columns per accumulator (48 used)
 constexpr uint32_t kTmemCols = kNAcc * kAccCols;
 constexpr uint32_t kIdesc = idesc_f16(128, kTokTile);
-constexpr unsigned long long kSpinLimitNs = 1000000000ull;
 constexpr int kRecvBytes = kRowsPerRank * kD * 4;  // merge partials one CTA sends another (fp32)
 constexpr int kRsBytes = 32 * kTokTile * 4;        // gate/up partials one CTA sends another (fp32)
 static_assert(kRecvBytes == kRsBytes, "the merge and the gate/up reduce-scatter share the receive buffer");
@@ -172,17 +171,20 @@ __device__ __forceinline__ void tmem_ld_sum4(uint32_t taddr, float (&v)[N]) {
     v[i] = ((__uint_as_float(r[0][i]) + __uint_as_float(r[1][i])) + __uint_as_float(r[2][i])) + __uint_as_float(r[3][i]);
 }
 
-// Bounded wait until *counter >= target (one thread polls, the CTA follows).
-// Once a wait of this CTA has timed out (*abort set), later waits return at
-// once, so a broken tick still ends within about a second per CTA.
-__device__ __forceinline__ void wait_counter(const int* counter, int target, int* status, volatile int* abort) {
+// Bounded wait until *counter >= target (one thread polls, the CTA follows), giving up
+// after limit_ns of globaltimer (checked after every failed poll: one poll is an L2 round
+// trip, far longer than the timer read). Once a wait of this CTA has timed out (*abort
+// set), later waits return at once, so a broken tick still ends within about a second
+// per CTA.
+__device__ __forceinline__ void wait_counter(const int* counter, int target, int* status, volatile int* abort,
+                                             unsigned long long limit_ns) {
   if (threadIdx.x == 0 && *abort == 0) {
     const unsigned long long t0 = global_timer_ns();
-    for (uint32_t it = 0;; ++it) {
+    for (;;) {
       int v;
       asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(counter) : "memory");
       if (v >= target) break;
-      if ((it & 63u) == 63u && global_timer_ns() - t0 > kSpinLimitNs) {
+      if (global_timer_ns() - t0 > limit_ns) {
         set_status(status, kStatusTimeout);
         *abort = 1;
         break;
@@ -207,7 +209,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   uint64_t* agbar = rsbar + 1;         // merged o_h rows of the partners
   uint64_t* bbar = agbar + 1;          // phase B: partial sums of x^2 and gate/up partials
   uint64_t* hbar = bbar + 1;           // phase B: the partners' SwiGLU columns
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(hbar + 1);
+  uint64_t* drain_bar = hbar + 1;      // the four issuing threads' last MMAs (before TMEM is freed)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);  // a wait of this CTA timed out
   float* gss = reinterpret_cast<float*>(smem + L.gss);
   float* rstd = reinterpret_cast<float*>(smem + L.rstd);
@@ -251,8 +254,10 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     const int i = q % kLayerChunks;
     return i >= kPersistAChunks + (in_b ? kPersistBChunks : 0);
   };
+  int issued_upto = 0;  // thread 0: ring positions issued so far (in increasing order)
   auto issue = [&](int q) {  // one thread; an empty position just completes the slot's phase
-    if (q >= total_chunks) return;
+    if (q >= total_chunks || *abort) return;  // after a timeout no new copy starts
+    issued_upto = q + 1;
     uint64_t* bar = full + (q % kSlots);
     if (is_empty(q)) {
       mbar_arrive(bar);
@@ -277,8 +282,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
   };
   uint32_t n_mma = 0;  // completed MMA groups (phase of mma_bar)
   // all threads: wait for the MMA groups just committed, then order TMEM reads after them
-  auto wait_mma = [&]() {
-    if (*abort == 0 && !mbar_wait(mma_bar, n_mma & 1u, p.status)) *abort = 1;
+  auto wait_mma = [&]() {  // this CTA's own MMAs always complete: waited even after a timeout
+    if (!mbar_wait(mma_bar, n_mma & 1u, p.status)) *abort = 1;
     ++n_mma;
     tc_fence_after();
   };
@@ -298,6 +303,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     for (int i = 0; i < kSlots; ++i) mbar_init(full + i, 1);
     mbar_init(mma_bar, kNAcc);
     for (int i = 0; i < kCl + 5; ++i) mbar_init(xbar + i, 1);
+    mbar_init(drain_bar, kNAcc);
     for (int q = 0; q < kSlots; ++q) issue(q);
   }
 
@@ -624,7 +630,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     const unsigned char* vc = n_chunks > 0 ? static_cast<const unsigned char*>(p.targs->v_cache[layer]) + head_off : nullptr;
 
     // =========================== phase A ===========================
-    wait_counter(p.counters + sA, sA == 0 ? G : n_b_ctas, p.status, abort);
+    wait_counter(p.counters + sA, sA == 0 ? G : n_b_ctas, p.status, abort, p.wait_limit_ns);
     {
       float4 xv[3][2];
       load_x(Xc, rank * 128, xv);
@@ -992,7 +998,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     // =========================== phase B ===========================
     if (in_b) {
       const int c = head;  // SwiGLU column block 64c..64c+63
-      wait_counter(p.counters + sA + 1, G, p.status, abort);
+      wait_counter(p.counters + sA + 1, G, p.status, abort, p.wait_limit_ns);
       {
         float4 xv[3][2];
         load_x(Xm, rank * 128, xv);
@@ -1113,10 +1119,15 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
     }
   }
 
-  // a tick that timed out may have skipped waits: let this CTA's last copies land
-  // (bounded) before the shared memory is released
-  if (tid == 0 && *abort)
-    for (int q = total_chunks - kSlots; q < total_chunks; ++q)
+  // ---- leave nothing in flight. Every path reaches this point, a timed-out tick included
+  // (its waits on other CTAs return at once). In order: this thread's cache-row copies;
+  // the ring copies issued (a timed-out tick stops issuing, and may have skipped the waits
+  // of the last ones: wait, bounded, for the last position of every slot); the MMAs of the
+  // four issuing threads (a last commit each on drain_bar); the partners' stores into this
+  // CTA's shared memory (the cluster barrier below); then the tensor memory is freed.
+  cp_async_wait<0>();
+  if (tid == 0)
+    for (int q = issued_upto - kSlots; q < issued_upto; ++q)
       if (q >= 0 && !is_empty(q)) {
         const unsigned long long t0 = global_timer_ns();
         uint32_t done = 0;
@@ -1127,6 +1138,12 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
               : "r"(smem_addr(full + q % kSlots)), "r"(static_cast<uint32_t>((q / kSlots) & 1))
               : "memory");
       }
+  if (warp < kNAcc) {
+    if (lane == 0) umma_commit(drain_bar);
+    __syncwarp();
+  }
+  mbar_wait(drain_bar, 0u, p.status);
+  tc_fence_after();
   // no CTA leaves while a partner may still write into its shared memory
   cluster.sync();
   tc_fence_before();
@@ -1136,7 +1153,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThr, 1) persisten
 
   // =========================== head ===========================
   if (cta == 0 && p.head) {
-    wait_counter(p.counters + 2 * p.n_layers, n_b_ctas, p.status, abort);
+    wait_counter(p.counters + 2 * p.n_layers, n_b_ctas, p.status, abort, p.wait_limit_ns);
     // a tick with a device-side error (an out-of-range cache value, a timeout) writes no waypoint
     if (*reinterpret_cast<volatile int*>(p.status) != 0) return;
     const float* Xf = X0 + static_cast<size_t>((2 * p.n_layers) % 3) * xs;

@@ -94,6 +94,7 @@ def _load():
         "fsx_get_status": (i32, [vp, vp]),
         "fsx_last_error": (ctypes.c_char_p, []),
         "fsx_destroy": (None, [vp]),
+        "fsx_set_wait_limit": (i32, [vp, ctypes.c_ulonglong]),
         "fsx_weight_bytes": (ctypes.c_longlong, [vp]),
         "fsx_tick_launches": (i32, [vp, i32]),
         "fsx_set_kernel_timing": (i32, [vp, i32, i32]),
@@ -150,7 +151,7 @@ def declared_symbols() -> list[str]:
             "fsx_append_get_status", "fsx_append_weight_bytes", "fsx_append_destroy", "fsx_append_set_concurrent",
             "fsx_session_create", "fsx_session_append", "fsx_session_tick", "fsx_session_committed",
             "fsx_session_reserved", "fsx_session_tick_stream", "fsx_session_append_stream", "fsx_session_sync",
-            "fsx_session_destroy"]
+            "fsx_session_destroy", "fsx_set_wait_limit"]
 
 
 def last_error() -> str:
@@ -260,6 +261,10 @@ class Expert:
 
     def weight_bytes(self) -> int:
         return int(lib().fsx_weight_bytes(self.h))
+
+    def set_wait_limit(self, ns: int):
+        """Test hook: limit of the single-launch tick's device-wide waits (0 = the default 1 s)."""
+        check(lib().fsx_set_wait_limit(self.h, ns))
 
     def launches(self, B: int) -> int:
         return int(lib().fsx_tick_launches(self.h, B))
