@@ -193,35 +193,26 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
 
   pdl_launch_dependents();
   pdl_wait();
-  if (*reinterpret_cast<volatile int*>(p.status) != 0) return;
   if ((smem_addr(smem) & 1023u) != 0u) {  // the swizzled operands need a 1024-byte aligned base
     if (tid == 0) set_status(p.status, kStatusDeviceArg);
     return;
   }
-  const int b = p.order != nullptr ? p.order[blockIdx.z] : static_cast<int>(blockIdx.z);
-
+  // Start-up is a chain of dependent global loads (vehicle, offsets, queries, own rows),
+  // each at the latency of a loaded memory system. The batched tick hands every CTA row
+  // its schedule entry (vehicle, first cache row, length: one load); the copies of the
+  // vehicle's queries and own keys / values are then in flight while the rest is read.
   const __nv_bfloat16* kc;
   const __nv_bfloat16* vc;
-  const int64_t* offs;
-  const int64_t* starts = nullptr;
   if (p.targs != nullptr) {
     kc = static_cast<const __nv_bfloat16*>(p.targs->k_cache[p.layer]);
     vc = static_cast<const __nv_bfloat16*>(p.targs->v_cache[p.layer]);
-    offs = p.targs->offsets;
-    starts = p.targs->starts;
   } else {
     kc = static_cast<const __nv_bfloat16*>(p.k_cache);
     vc = static_cast<const __nv_bfloat16*>(p.v_cache);
-    offs = p.offsets;
   }
-  const long long o_lo = starts != nullptr ? starts[b] : offs[b];
-  const long long o_hi = o_lo + (offs[b + 1] - offs[b]);
-  if (o_lo < 0 || o_hi < o_lo || o_hi > p.max_total || (o_hi > o_lo && (kc == nullptr || vc == nullptr))) {
-    set_status(p.status, kStatusDeviceArg);  // never read outside the caller's cache
-    return;
-  }
-  const long long L = o_hi - o_lo;
-  const int n_chunks = 1 + static_cast<int>((L + kSlotKeys - 1) / kSlotKeys);  // chunk 0: own keys
+  AttnPlan plan_z{0, 0, 0};
+  if (p.plan != nullptr) plan_z = p.plan[blockIdx.z];
+  const int b = p.plan != nullptr ? plan_z.b : (p.order != nullptr ? p.order[blockIdx.z] : static_cast<int>(blockIdx.z));
 
   unsigned char* qt = smem + kOffQ;
   unsigned char* kslot = smem + kOffK;
@@ -238,30 +229,6 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kNumBars);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-  if (tid == 0) {
-    for (int i = 0; i < kSlots; ++i) {
-      mbar_init(kfull + i, kProdThreads);
-      mbar_init(kempty + i, 1);
-      mbar_init(vfull + i, kProdThreads);
-      mbar_init(vempty + i, 1);
-      mbar_arrive(kempty + i);  // release 0 of every slot: free from the start
-      mbar_arrive(vempty + i);
-    }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(sfull + i, 1);
-      mbar_init(pfull + i, kSoftmaxWarps * 32);
-      mbar_init(pvdone + i, 1);
-    }
-    mbar_init(drain, 1);
-    *abort = 0;
-  }
-  if (warp == kMmaWarp) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(tmem_slot)),
-                 "r"(kTmemCols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-  }
-
   // ---- producers' staging of chunk i (own rows fp16, cache rows bf16 converted later)
   const bool is_prod = warp >= kProdWarp0;
   const bool is_v = warp >= kProdWarp0 + 2;
@@ -269,8 +236,9 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
   const int pu = pt & 15;                 // 16-byte unit of a 256-byte row
   const int pr0 = pt >> 4;                // rows pr0, pr0 + 4, ...
   const size_t tok = static_cast<size_t>(H) * kD;
-  const __nv_bfloat16* cbase = (is_v ? vc : kc) + (static_cast<size_t>(o_lo) * H + h) * kD + pu * 8;
   const __half* obase = (is_v ? p.v_own : p.k_own) + static_cast<size_t>(b) * p.n_own * p.own_stride + h * kD + pu * 8;
+  const __nv_bfloat16* cbase = nullptr;  // this CTA's first cache row of the tensor, set below
+  long long L = 0;
   unsigned char* pslots = is_v ? vslot : kslot;
   auto chunk_rows = [&](int i) {
     return i == 0 ? p.n_own
@@ -294,23 +262,83 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
     }
     cp_async_commit();
   };
-  if (is_prod) {  // chunks 0 and 1 are in flight while Q is staged
-    issue(0);
-    if (n_chunks > 1) issue(1);
-  }
-  for (int i = tid; i < 64 * 16; i += kThreadsTc) {  // Q: 64 rows x 16 units (rows >= n_q zero)
+  // queries: 64 rows x 16 units, rows >= n_q zero (one copy group per thread)
+  for (int i = tid; i < 64 * 16; i += kThreadsTc) {
     const int r = i >> 4;
     const int u = i & 15;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    unsigned char* dst = qt + tile128_off(r, u);
     if (r < p.n_q)
-      v = *reinterpret_cast<const uint4*>(p.q + (static_cast<size_t>(b) * p.n_q + r) * p.q_stride + h * kD + u * 8);
-    *reinterpret_cast<uint4*>(qt + tile128_off(r, u)) = v;
+      cp_async_16(smem_addr(dst), p.q + (static_cast<size_t>(b) * p.n_q + r) * p.q_stride + h * kD + u * 8);
+    else
+      *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
+  }
+  cp_async_commit();
+  if (is_prod) issue(0);  // own keys / values
+
+  long long o_lo, o_hi;
+  if (p.plan != nullptr) {
+    o_lo = plan_z.lo;
+    o_hi = o_lo + plan_z.len;  // a length of -1 fails the check below
+  } else {
+    const int64_t* offs = p.targs != nullptr ? p.targs->offsets : p.offsets;
+    const int64_t* starts = p.targs != nullptr ? p.targs->starts : nullptr;
+    o_lo = starts != nullptr ? starts[b] : offs[b];
+    o_hi = o_lo + (offs[b + 1] - offs[b]);
+  }
+  if (o_lo < 0 || o_hi < o_lo || o_hi > p.max_total || (o_hi > o_lo && (kc == nullptr || vc == nullptr))) {
+    cp_async_wait<0>();  // the query / own-row copies land before the CTA leaves
+    set_status(p.status, kStatusDeviceArg);  // never read outside the caller's cache
+    return;
+  }
+  L = o_hi - o_lo;
+  const int n_chunks = 1 + static_cast<int>((L + kSlotKeys - 1) / kSlotKeys);  // chunk 0: own keys
+  cbase = (is_v ? vc : kc) + (static_cast<size_t>(o_lo) * H + h) * kD + pu * 8;
+
+  if (tid == 0) {
+    for (int i = 0; i < kSlots; ++i) {
+      mbar_init(kfull + i, kProdThreads);
+      mbar_init(kempty + i, 1);
+      mbar_init(vfull + i, kProdThreads);
+      mbar_init(vempty + i, 1);
+      mbar_arrive(kempty + i);  // release 0 of every slot: free from the start
+      mbar_arrive(vempty + i);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(sfull + i, 1);
+      mbar_init(pfull + i, kSoftmaxWarps * 32);
+      mbar_init(pvdone + i, 1);
+    }
+    mbar_init(drain, 1);
+    // a kernel before this one has already abandoned the tick: this CTA stops below
+    *abort = *reinterpret_cast<volatile int*>(p.status) != 0 ? 1 : 0;
+  }
+  if (warp == kMmaWarp) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(tmem_slot)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  if (is_prod) {  // the first cache chunk; then wait for this thread's query copies
+    if (n_chunks > 1) {
+      issue(1);
+      cp_async_wait<2>();
+    } else {
+      cp_async_wait<1>();
+    }
+  } else {
+    cp_async_wait<0>();
   }
   fence_proxy_async();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(tmem_slot);
+  if (*abort) {  // the tick was abandoned before this kernel: no MMA was issued
+    cp_async_wait<0>();
+    if (warp == kMmaWarp)
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+    return;
+  }
 
   if (warp == kMmaWarp) {
     // ---------------------------------------------------------------- MMA issuer

@@ -50,6 +50,13 @@ __global__ void embed_kernel(const EmbedArgs a) {
       int r = 0;
       for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) r += s_cnt[w];
       a.order[r] = row;
+      if (a.plan != nullptr) {
+        AttnPlan e;
+        e.lo = a.targs->starts != nullptr ? a.targs->starts[row] : off[row];
+        e.b = row;
+        e.len = (len >= 0 && len <= 0x7fffffff) ? static_cast<int>(len) : -1;
+        a.plan[r] = e;
+      }
     }
   }
   float* xr = a.x + static_cast<size_t>(row) * a.d;

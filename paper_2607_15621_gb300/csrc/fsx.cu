@@ -86,6 +86,7 @@ struct fsx_handle_s {
   float* gemm_part = nullptr;   // split-K partial tiles of the residual GEMMs
   int* tile_count = nullptr;    // [sm_count] split arrivals per tile, zero between launches
   int* order = nullptr;         // [max_batch] vehicles by decreasing cache length (attention schedule)
+  fsx::AttnPlan* plan = nullptr;  // [max_batch] the same schedule with each vehicle's cache range
   int* status = nullptr;
   TickArgs* d_args = nullptr;
   TickArgs h_args{};
@@ -249,6 +250,7 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
   ea.ss = h->ss;
   ea.ss_stride = h->ss_stride;
   ea.order = h->order;
+  ea.plan = h->plan;
   ea.status = h->status;
   FSX_CUDA(fsx::launch_embed(ea, st, pdl));
 
@@ -299,6 +301,7 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     a.part_o = h->part;
     a.part_lse = h->part + static_cast<size_t>(B) * c.n_heads * S * fsx::kTokTile * fsx::kHeadDim;
     a.order = h->order;
+    a.plan = h->plan;
     a.status = h->status;
     FSX_CUDA(mark(kClassAttn, true));
     FSX_CUDA(fsx::launch_attention(a, B, c.cache_dtype, st, pdl));
@@ -473,7 +476,7 @@ void free_handle(fsx_handle_s* h) {
   if (h->paper_params) cudaFree(h->paper_params);
   if (h->paper_frames) cudaFree(h->paper_frames);
   void* bufs[] = {h->p_arena, h->p_x, h->p_counters, h->w_arena, h->params, h->x, h->x16, h->ss, h->qkv, h->o, h->hbuf, h->part,
-                  h->gemm_part, h->tile_count, h->order, h->status, h->d_args,
+                  h->gemm_part, h->tile_count, h->order, h->plan, h->status, h->d_args,
                   h->st_offsets, h->st_frames, h->st_waypoints};
   for (void* p : bufs)
     if (p) cudaFree(p);
@@ -750,6 +753,7 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
   FSX_CUDA_H(cudaMalloc(&h->tile_count, sizeof(int) * h->sm_count));
   FSX_CUDA_H(cudaMemset(h->tile_count, 0, sizeof(int) * h->sm_count));
   FSX_CUDA_H(cudaMalloc(&h->order, sizeof(int) * cfg->max_batch));
+  FSX_CUDA_H(cudaMalloc(&h->plan, sizeof(fsx::AttnPlan) * cfg->max_batch));
   FSX_CUDA_H(cudaMalloc(&h->status, sizeof(int)));
   FSX_CUDA_H(cudaMemset(h->status, 0, sizeof(int)));
   FSX_CUDA_H(cudaMalloc(&h->d_args, sizeof(TickArgs)));

@@ -337,49 +337,68 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
             // token pairs (j, j + 1): the even lane packs columns (row, row + 1) of token j,
             // the odd lane columns (row - 1, row) of token j + 1 -- one two-value fp16
             // conversion and one 4-byte store per pair instead of two of each
+            // (the sixteen exchanges are issued together, then the conversions and stores:
+            // independent chains, so their latencies overlap)
             const bool odd = (lane & 1) != 0;
+            float v[32];
 #pragma unroll
-            for (int j = 0; j < 32; j += 2) {
-              float a = __uint_as_float(r[j]);
-              float b = __uint_as_float(r[j + 1]);
-              if (NORM) {
-                a *= rs[j];
-                b *= rs[j + 1];
-              }
-              const float other = __shfl_xor_sync(0xffffffffu, odd ? a : b, 1);
-              const __half2 h2 = odd ? __floats2half2_rn(other, b) : __floats2half2_rn(a, other);
-              *reinterpret_cast<__half2*>(tH + (odd ? (j + 1) * kSH + row - 1 : j * kSH + row)) = h2;
-            }
+            for (int j = 0; j < 32; ++j) v[j] = NORM ? __uint_as_float(r[j]) * rs[j] : __uint_as_float(r[j]);
+            float other[16];
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj)
+              other[jj] = __shfl_xor_sync(0xffffffffu, odd ? v[2 * jj] : v[2 * jj + 1], 1);
+            // token 2jj (even lane) or 2jj + 1 (odd lane), columns from row & ~1
+            __half2* dst = reinterpret_cast<__half2*>(tH + (odd ? kSH + row - 1 : row));
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj)
+              dst[jj * kSH] = odd ? __floats2half2_rn(other[jj], v[2 * jj + 1]) : __floats2half2_rn(v[2 * jj], other[jj]);
           }
+          if (EPI == kEpiSwiglu) {
+            // SwiGLU: lane l (l % 16 < 8) holds a gate row, lane l + 8 its up row; every
+            // exchange first, then the activations and stores
+            float v[32], up[32];
 #pragma unroll
-          for (int j = 0; j < 32 && EPI == kEpiSwiglu; ++j) {
-            float val = __uint_as_float(r[j]);
-            if (NORM) val *= rs[j];
-            {  // SwiGLU: lane l (l % 16 < 8) holds a gate row, lane l + 8 its up row
-              const float up = __shfl_down_sync(0xffffffffu, val, 8);
-              const __half hv = __float2half_rn(__fdividef(val, 1.f + __expf(-val)) * up);
-              if ((lane & 8) == 0) tH[j * kSG + (row >> 4) * 8 + (lane & 7)] = hv;
+            for (int j = 0; j < 32; ++j) v[j] = NORM ? __uint_as_float(r[j]) * rs[j] : __uint_as_float(r[j]);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) up[j] = __shfl_down_sync(0xffffffffu, v[j], 8);
+            __half* dst = tH + (row >> 4) * 8 + (lane & 7);
+            if ((lane & 8) == 0) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) dst[j * kSG] = __float2half_rn(__fdividef(v[j], 1.f + __expf(-v[j])) * up[j]);
             }
           }
           half_sync(half);
           // coalesced 16-byte stores of the chunk's token rows
-          if (EPI == kEpiStore) {
-            for (int e = htid; e < nc * (kTileN / 8); e += 128) {
-              const int tk = e / (kTileN / 8);
-              const int u = e % (kTileN / 8);
-              const int m = m0 + c0 + tk;
-              if (m < p.M)
-                *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m) * p.ldy + n0 + u * 8) =
-                    *reinterpret_cast<const uint4*>(tH + tk * kSH + u * 8);
+          // (all of a thread's staging reads before its first global store)
+          if (EPI == kEpiStore) {  // 32 tokens x 16 units: four per thread
+            uint4 val[4];
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              const int e = htid + t * 128;
+              val[t] = *reinterpret_cast<const uint4*>(tH + (e >> 4) * kSH + (e & 15) * 8);
             }
-          } else {
-            for (int e = htid; e < nc * 8; e += 128) {
-              const int tk = e >> 3;
-              const int u = e & 7;
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              const int e = htid + t * 128;
+              const int tk = e >> 4;
               const int m = m0 + c0 + tk;
-              if (m < p.M)
-                *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m) * p.ldy + n0 / 2 + u * 8) =
-                    *reinterpret_cast<const uint4*>(tH + tk * kSG + u * 8);
+              if (tk < nc && m < p.M)
+                *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m) * p.ldy + n0 + (e & 15) * 8) = val[t];
+            }
+          } else {  // 32 tokens x 8 units: two per thread
+            uint4 val[2];
+#pragma unroll
+            for (int t = 0; t < 2; ++t) {
+              const int e = htid + t * 128;
+              val[t] = *reinterpret_cast<const uint4*>(tH + (e >> 3) * kSG + (e & 7) * 8);
+            }
+#pragma unroll
+            for (int t = 0; t < 2; ++t) {
+              const int e = htid + t * 128;
+              const int tk = e >> 3;
+              const int m = m0 + c0 + tk;
+              if (tk < nc && m < p.M)
+                *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m) * p.ldy + n0 / 2 + (e & 7) * 8) = val[t];
             }
           }
           half_sync(half);  // staging free for the next chunk

@@ -32,6 +32,14 @@ struct TickArgs {
 enum GemmEpilogue { kEpiStore = 0, kEpiResidual = 1, kEpiSwiglu = 2 };
 
 // ------------------------------------------------------------- attention
+// Entry z of the batched tick's attention schedule (written by the embed kernel in
+// longest-cache-first order): vehicle b, its first cache row and its number of rows.
+struct AttnPlan {
+  long long lo;
+  int b;
+  int len;  // -1 when the caller's offsets give no valid length
+};
+
 struct AttnArgs {
   const __half* q;
   long long q_stride;
@@ -54,6 +62,7 @@ struct AttnArgs {
   float* part_o;              // [B, H, S, 48, 128] when n_splits > 1
   float* part_lse;            // [B, H, S, 48]   (log2 domain)
   const int* order;           // optional [B]: CTA row z works on vehicle order[z] (longest cache first)
+  const AttnPlan* plan;       // optional [B] (tensor-core path): CTA row z works on plan[z]
   int* status;
 };
 
@@ -80,6 +89,7 @@ struct EmbedArgs {
   float* ss;              // per-row sums of x^2 over 128-column groups, [d/128][ss_stride]
   int ss_stride;
   int* order;             // optional [B]: vehicles by decreasing cache length (ties by index)
+  AttnPlan* plan;         // optional [B]: the same order with each vehicle's cache range
   int* status;
 };
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t stream, bool pdl);
