@@ -68,7 +68,7 @@ struct fsx_handle_s {
   long long weight_bytes = 0;
   std::vector<const unsigned char*> w_qkv, w_o, w_gu, w_dn;  // tcgen05 tile images per layer
   // 2-D tensor maps of the activation buffers for the token tile sizes 48 / 128 / 256
-  CUtensorMap map_x16[3], map_o[3], map_h[3];
+  CUtensorMap map_x16[4], map_o[4], map_h[4];  // token boxes of 48, 128, 256, 144 rows
   // fp32 small parameters
   float* params = nullptr;
   float *act_emb = nullptr, *pos_emb = nullptr, *attn_norm = nullptr, *mlp_norm = nullptr;
@@ -262,6 +262,11 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
   // tcgen05.mma costs the same for any N up to 256) whenever M exceeds one 48-token tile
   const int bq_i = M <= 48 ? 0 : 2;
   const int bq = bq_i == 0 ? 48 : 256;
+  // The residual GEMMs (N = d) have only d / 128 weight tiles: with 256-token tiles they
+  // fill about half the SMs. 144-token tiles give one tile per SM up to 38 x 144 tokens.
+  const int rtiles144 = (d / 128) * ((M + 143) / 144);
+  const int rbn_i = (bn_i == 2 && rtiles144 <= h->sm_count) ? 3 : bn_i;
+  const int rbn = rbn_i == 3 ? 144 : bn;
   const int S = attention_splits(h, B);
 
   for (int l = 0; l < c.n_layers; ++l) {
@@ -323,11 +328,11 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     go.ldxo = d;
     go.ss_out = h->ss;
     go.ss_stride = h->ss_stride;
-    go.k_splits = fsx::gemm_tc_k_splits((d / 128) * ((M + bn - 1) / bn), HD / 64, h->sm_count);
+    go.k_splits = fsx::gemm_tc_k_splits((d / 128) * ((M + rbn - 1) / rbn), HD / 64, h->sm_count);
     go.part = h->gemm_part;
     go.tile_count = h->tile_count;
     FSX_CUDA(mark(kClassWo, true));
-    FSX_CUDA(fsx::launch_gemm_tc(h->map_o[bn_i], go, bn, fsx::kEpiResidual, false, st, pdl));
+    FSX_CUDA(fsx::launch_gemm_tc(h->map_o[rbn_i], go, rbn, fsx::kEpiResidual, false, st, pdl));
     FSX_CUDA(mark(kClassWo, false));
 
     // h = silu(RMSNorm(x) W_g^T) * (RMSNorm(x) W_u^T)
@@ -358,11 +363,11 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     gd.ldxo = d;
     gd.ss_out = h->ss;
     gd.ss_stride = h->ss_stride;
-    gd.k_splits = fsx::gemm_tc_k_splits((d / 128) * ((M + bn - 1) / bn), F / 64, h->sm_count);
+    gd.k_splits = fsx::gemm_tc_k_splits((d / 128) * ((M + rbn - 1) / rbn), F / 64, h->sm_count);
     gd.part = h->gemm_part;
     gd.tile_count = h->tile_count;
     FSX_CUDA(mark(kClassDown, true));
-    FSX_CUDA(fsx::launch_gemm_tc(h->map_h[bn_i], gd, bn, fsx::kEpiResidual, false, st, pdl));
+    FSX_CUDA(fsx::launch_gemm_tc(h->map_h[rbn_i], gd, rbn, fsx::kEpiResidual, false, st, pdl));
     FSX_CUDA(mark(kClassDown, false));
   }
 
@@ -736,8 +741,8 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
   FSX_CUDA_H(cudaMemset(h->o, 0, m_pad * HD * sizeof(__half)));
   FSX_CUDA_H(cudaMemset(h->hbuf, 0, m_pad * F * sizeof(__half)));
   {
-    const uint32_t boxes[3] = {48, 128, 256};
-    for (int i = 0; i < 3; ++i) {
+    const uint32_t boxes[4] = {48, 128, 256, 144};
+    for (int i = 0; i < 4; ++i) {
       if (!fsx::encode_act_map(&h->map_x16[i], h->x16, m_pad, d, boxes[i]) ||
           !fsx::encode_act_map(&h->map_o[i], h->o, m_pad, HD, boxes[i]) ||
           !fsx::encode_act_map(&h->map_h[i], h->hbuf, m_pad, F, boxes[i]))

@@ -37,7 +37,6 @@ namespace {
 constexpr int kEpiGroups = 3;         // epilogue groups of 4 warps (one per TMEM lane quadrant)
 constexpr int kEpiThreads = kEpiGroups * 128;
 constexpr int kTcThreads = 64 + kEpiThreads;  // producer warp, MMA warp, epilogue groups
-constexpr int kStages = 4;
 constexpr int kTileN = 128;           // weight rows per tile (MMA M)
 constexpr int kTileK = 64;            // K per stage (128 bytes of fp16: one swizzle span)
 constexpr int kWTileBytes = kTileN * kTileK * 2;  // 16 KB
@@ -62,6 +61,15 @@ __host__ __device__ constexpr int tc_stage_bytes() {
   return kWTileBytes + BN * kTileK * 2;
 }
 
+// Depth of the stage ring. A stage stays in flight for a round trip set by the L2 / HBM
+// latency under load (copy issue, transfer, MMAs, release), so the ring takes as many
+// stages as the shared memory holds: 4 of 48 KB for 256-token tiles, 5 of 34 KB for 144,
+// 6 of 32 KB for 128, 8 of 22 KB for 48.
+template <int BN>
+__host__ __device__ constexpr int tc_stages() {
+  return BN >= 256 ? 4 : (BN >= 144 ? 5 : (BN >= 128 ? 6 : 8));
+}
+
 template <int BN>
 __host__ __device__ constexpr int tc_rstd_bytes() {  // 1/rms of the tokens, double-buffered by tile parity
   return ((2 * BN * 4 + 1023) / 1024) * 1024;
@@ -73,10 +81,13 @@ static_assert(kStgHalfBytes % 1024 == 0 && kSspBytes % 1024 == 0, "the stage rin
 template <int BN>
 __host__ __device__ constexpr int tc_smem_bytes() {
   return 1024 /* barriers, tmem address */ + tc_rstd_bytes<BN>() + kSspBytes + kEpiGroups * kStgHalfBytes +
-         1024 /* alignment slack */ + kStages * tc_stage_bytes<BN>();
+         1024 /* alignment slack */ + tc_stages<BN>() * tc_stage_bytes<BN>();
 }
 
-static_assert(tc_smem_bytes<256>() <= 232448, "shared memory of the widest tile exceeds the per-block limit");
+static_assert(tc_smem_bytes<256>() <= 232448 && tc_smem_bytes<144>() <= 232448 && tc_smem_bytes<128>() <= 232448 &&
+                  tc_smem_bytes<48>() <= 232448,
+              "shared memory of a tile shape exceeds the per-block limit");
+static_assert(2 * 8 * 8 + 2 * 2 * 8 + 8 <= 1024, "barriers of the deepest ring exceed the header");
 
 template <int BN>
 __host__ __device__ constexpr uint32_t tc_tmem_cols() {  // two accumulators, power of two >= 32
@@ -87,6 +98,7 @@ template <int BN, int EPI, bool NORM>
 __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_constant__ CUtensorMap map_a,
                                                                const TcGemmArgs p) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
+  constexpr int kStages = tc_stages<BN>();
   // 1024-byte aligned stage area (the swizzle pattern repeats every 1024 bytes)
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -507,6 +519,7 @@ const void* tc_select(int bn, int epi, bool norm, size_t* smem) {
   FSX_TC(128, kEpiStore, true)
   FSX_TC(128, kEpiSwiglu, true)
   FSX_TC(128, kEpiResidual, false)
+  FSX_TC(144, kEpiResidual, false)
   FSX_TC(256, kEpiStore, true)
   FSX_TC(256, kEpiSwiglu, true)
   FSX_TC(256, kEpiResidual, false)
@@ -517,7 +530,7 @@ const void* tc_select(int bn, int epi, bool norm, size_t* smem) {
 }  // namespace
 
 cudaError_t gemm_tc_set_attributes() {
-  const int bns[3] = {48, 128, 256};
+  const int bns[4] = {48, 128, 144, 256};
   const int epis[3] = {kEpiStore, kEpiSwiglu, kEpiResidual};
   for (int bn : bns)
     for (int epi : epis)
