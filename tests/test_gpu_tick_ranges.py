@@ -104,10 +104,13 @@ def test_staleness_clip_forward_matches_the_oracle():
         _check(wp, att, j, ref_wp[j], ref_att[j], SMALL.n_tok)
 
 
+@pytest.mark.parametrize("case", ["past_end", "negative_start", "decreasing_offsets"])
 @pytest.mark.parametrize("B", [1, 2])
-def test_ranges_outside_the_cache_are_rejected(B):
-    """A start row whose range runs past max_total_cache_tokens sets the status word and
-    the tick writes no waypoint (the single-launch and the graph path)."""
+def test_ranges_outside_the_cache_are_rejected(B, case):
+    """A range the cache does not hold sets the status word and the tick writes no
+    waypoint (the single-launch and the graph path): a start row whose range runs past
+    max_total_cache_tokens, a negative start row, and offsets that decrease (a negative
+    length) while start rows are given."""
     rows = 100
     k, v, _ = synth.make_cache(SMALL, [rows], 14, "bf16")
     k = [t.cuda() for t in k]
@@ -116,13 +119,21 @@ def test_ranges_outside_the_cache_are_rejected(B):
     w = fc.weights(SMALL, 14, "bf16")
     ex = fsx.Expert(SMALL, w, B, rows, "bf16", "bf16")
     try:
-        off = torch.tensor([0] + [20 * (i + 1) for i in range(B)], dtype=torch.int64, device="cuda")
-        starts = torch.tensor([90] + [0] * (B - 1), dtype=torch.int64, device="cuda")
+        good_off = [0] + [20 * (i + 1) for i in range(B)]
+        if case == "past_end":  # vehicle 0 reads rows 90 .. 109 of a 100-row cache
+            off_l, starts_l = good_off, [90] + [0] * (B - 1)
+        elif case == "negative_start":
+            off_l, starts_l = good_off, [-4] + [0] * (B - 1)
+        else:  # the last vehicle's length is -10
+            off_l, starts_l = good_off[:-1] + [good_off[-2] - 10], [0] * B
+        off = torch.tensor(off_l, dtype=torch.int64, device="cuda")
+        starts = torch.tensor(starts_l, dtype=torch.int64, device="cuda")
         out = torch.full((B, SMALL.n_waypoints, 2), 123.0, device="cuda")
         ex.tick(k, v, off, frames, out, starts=starts)
         assert ex.status() == fsx.FSX_ERR_DEVICE_ARG
         assert torch.all(out == 123.0)
         ok = torch.zeros(B, dtype=torch.int64, device="cuda")
+        off = torch.tensor(good_off, dtype=torch.int64, device="cuda")
         wp, _ = _tick(ex, k, v, off, frames, starts=ok)
         assert np.isfinite(wp).all()
     finally:
