@@ -25,6 +25,7 @@
 // ready; warps 4-5 stage (and convert) the K rows, warps 6-7 the V rows, two chunks ahead.
 // Every wait is bounded; a timeout raises the status word and the CTA drains its
 // MMAs before it frees the tensor memory.
+#include <cuda.h>
 #include <math_constants.h>
 
 #include "device_util.cuh"
@@ -54,8 +55,8 @@ constexpr int kOffQ = 0;
 constexpr int kOffK = kOffQ + kQBytes;
 constexpr int kOffV = kOffK + kSlots * kSlotBytes;
 constexpr int kOffBar = kOffV + kSlots * kSlotBytes;
-// barriers: kfull[3], kempty[3], vfull[3], vempty[3], sfull[2], pfull[2], pvdone[2], drain
-constexpr int kNumBars = 19;
+// barriers: kfull[3], kempty[3], vfull[3], vempty[3], sfull[2], pfull[2], pvdone[2], drain, ktma[3], vtma[3]
+constexpr int kNumBars = 25;
 constexpr int kSmemTc = kOffBar + kNumBars * 8 + 8 /*tmem slot + abort*/;
 static_assert(kSmemTc + 1024 <= (228 * 1024) / 2, "two CTAs per SM");
 
@@ -183,6 +184,16 @@ __device__ __forceinline__ void tmem_st_16x128b_x8(uint32_t taddr, const uint32_
 
 constexpr float kLazyRescale = 8.f;  // log2 units; P <= 2^8 between rescales
 
+// one 64-token x 64-dim box of a head of the cache (3-D map [rows, heads, 128], 128-byte swizzle)
+__device__ __forceinline__ void tma_load_cache(void* dst, const CUtensorMap* map, int x, int head, int row,
+                                               uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+      "[%5];" ::"r"(smem_addr(dst)),
+      "l"(map), "r"(x), "r"(head), "r"(row), "r"(smem_addr(bar))
+      : "memory");
+}
+
 __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p) {
   extern __shared__ __align__(1024) unsigned char smem[];
   const int tid = threadIdx.x;
@@ -226,6 +237,8 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
   uint64_t* pfull = bars + 14;   // [2] P of a chunk written over its S
   uint64_t* pvdone = bars + 16;  // [2] P V of a chunk done (one per buffer)
   uint64_t* drain = bars + 18;   // every MMA of the CTA done
+  uint64_t* ktma = bars + 19;    // [3] a whole cache chunk's K rows landed by TMA
+  uint64_t* vtma = bars + 22;    // [3] the same for V
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kNumBars);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -239,7 +252,18 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
   const __half* obase = (is_v ? p.v_own : p.k_own) + static_cast<size_t>(b) * p.n_own * p.own_stride + h * kD + pu * 8;
   const __nv_bfloat16* cbase = nullptr;  // this CTA's first cache row of the tensor, set below
   long long L = 0;
+  long long row0 = 0;                    // this CTA's first cache row, set below
   unsigned char* pslots = is_v ? vslot : kslot;
+  // Whole cache chunks (every cache chunk but a short last one) come by two TMA box loads
+  // issued by one thread of the tensor's warps (when the batched tick supplies the cache
+  // maps); the own keys and a short last chunk by 16-byte copies of every thread.
+  const CUtensorMap* tmap =
+      (p.cache_maps != nullptr && p.targs != nullptr) ? p.cache_maps + 2 * p.layer + (is_v ? 1 : 0) : nullptr;
+  uint64_t* tbar = is_v ? vtma : ktma;
+  auto by_tma = [&](int i) { return tmap != nullptr && i >= 1 && static_cast<long long>(i) * kSlotKeys <= L; };
+  // chunks 1 .. L / 64 are the TMA chunks, so slot s = i mod 3 sees them in order from its
+  // first one (i = 3 for slot 0): the phase of chunk i on its slot's barrier
+  auto tma_parity = [](int i) { return static_cast<uint32_t>((i / kSlots - (i % kSlots == 0 ? 1 : 0)) & 1); };
   auto chunk_rows = [&](int i) {
     return i == 0 ? p.n_own
                   : static_cast<int>(min(static_cast<long long>(kSlotKeys), L - (i - 1) * static_cast<long long>(kSlotKeys)));
@@ -248,6 +272,17 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
     unsigned char* slot = pslots + (i % kSlots) * kSlotBytes;
     const int rows = chunk_rows(i);
     const long long c0 = (i - 1) * static_cast<long long>(kSlotKeys);
+    if (by_tma(i)) {
+      if (pt == 0) {
+        uint64_t* bar = tbar + i % kSlots;
+        const int y = static_cast<int>(row0 + c0);
+        mbar_arrive_expect_tx(bar, kSlotBytes);
+        tma_load_cache(slot, tmap, 0, h, y, bar);
+        tma_load_cache(slot + kSlotBytes / 2, tmap, 64, h, y, bar);
+      }
+      cp_async_commit();  // an empty group keeps one group per chunk
+      return;
+    }
 #pragma unroll 8
     for (int m = 0; m < kSlotKeys / 4; ++m) {
       const int r = pr0 + 4 * m;
@@ -291,6 +326,7 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
     return;
   }
   L = o_hi - o_lo;
+  row0 = o_lo;
   const int n_chunks = 1 + static_cast<int>((L + kSlotKeys - 1) / kSlotKeys);  // chunk 0: own keys
   cbase = (is_v ? vc : kc) + (static_cast<size_t>(o_lo) * H + h) * kD + pu * 8;
 
@@ -319,6 +355,10 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   if (is_prod) {  // the first cache chunk; then wait for this thread's query copies
+    if (pt == 0 && tmap != nullptr) {  // the TMA barriers, before the first TMA chunk; read after the CTA barrier
+      for (int i = 0; i < kSlots; ++i) mbar_init(tbar + i, 1);
+      fence_proxy_async();
+    }
     if (n_chunks > 1) {
       issue(1);
       cp_async_wait<2>();
@@ -335,6 +375,7 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(tmem_slot);
   if (*abort) {  // the tick was abandoned before this kernel: no MMA was issued
     cp_async_wait<0>();
+    if (is_prod && pt == 0 && n_chunks > 1 && by_tma(1)) mbar_wait(tbar + 1, 0, p.status);  // chunk 1 landed
     if (warp == kMmaWarp)
       asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
     return;
@@ -418,14 +459,23 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
     uint64_t* full = is_v ? vfull : kfull;
     uint64_t* empty = is_v ? vempty : kempty;
     bool ok = true;
-    for (int i = 0; ok && i < n_chunks; ++i) {
+    int issued = n_chunks > 1 ? 2 : 1;  // chunks whose loads were issued
+    int i = 0;
+    for (; ok && i < n_chunks; ++i) {
       if (i + 1 < n_chunks) cp_async_wait<1>();
       else cp_async_wait<0>();
+      if (by_tma(i)) {
+        ok = wait_bar(tbar + i % kSlots, tma_parity(i), p.status, abort);
+        if (!ok) break;
+      }
       // refill first when the slot of chunk i - 1 is already free (the warp agrees on it)
       bool refilled = false;
       if (i + 2 < n_chunks) {
         refilled = __all_sync(0xffffffffu, test_bar(empty + ((i + 2) % kSlots), ((i + 2) / kSlots) & 1));
-        if (refilled) issue(i + 2);
+        if (refilled) {
+          issue(i + 2);
+          issued = i + 3;
+        }
       }
       if (i > 0 && !is_v) {  // cache K rows -> fp16 (V stays bf16)
         unsigned char* slot = pslots + (i % kSlots) * kSlotBytes;
@@ -440,10 +490,17 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
       mbar_arrive(full + (i % kSlots));
       if (i + 2 < n_chunks && !refilled) {
         ok = wait_bar(empty + ((i + 2) % kSlots), ((i + 2) / kSlots) & 1, p.status, abort);
-        if (ok) issue(i + 2);
+        if (ok) {
+          issue(i + 2);
+          issued = i + 3;
+        }
       }
     }
     cp_async_wait<0>();
+    // after an abort: the TMA chunks issued but not consumed land before the CTA leaves
+    if (pt == 0)
+      for (int j = i; j < issued; ++j)
+        if (by_tma(j)) mbar_wait(tbar + j % kSlots, tma_parity(j), p.status);
   } else {
     // ---------------------------------------------------------------- softmax rows
     // Warp w owns query rows 16 w .. 16 w + 15 (tensor-memory lanes 32 w .. + 15).

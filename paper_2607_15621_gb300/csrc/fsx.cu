@@ -91,6 +91,10 @@ struct fsx_handle_s {
   TickArgs* d_args = nullptr;
   TickArgs h_args{};
   bool args_valid = false;
+  // bf16 caches: TMA maps of every layer's K and V cache ([2 n_layers], device), re-encoded
+  // whenever the cache pointers change; the tensor-core attention loads whole chunks with them
+  CUtensorMap* d_cache_maps = nullptr;
+  std::vector<CUtensorMap> h_cache_maps;
   // persistent single-vehicle tick
   bool persist_ok = false;
   void* p_arena = nullptr;
@@ -307,6 +311,7 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
     a.part_lse = h->part + static_cast<size_t>(B) * c.n_heads * S * fsx::kTokTile * fsx::kHeadDim;
     a.order = h->order;
     a.plan = h->plan;
+    a.cache_maps = h->d_cache_maps;
     a.status = h->status;
     FSX_CUDA(mark(kClassAttn, true));
     FSX_CUDA(fsx::launch_attention(a, B, c.cache_dtype, st, pdl));
@@ -455,8 +460,24 @@ fsx_status prepare_tick(fsx_handle_s* h, const void* const* k_cache, const void*
   a.frames = d_frames;
   a.waypoints = d_waypoints;
   if (!h->args_valid || std::memcmp(&a, &h->h_args, sizeof(TickArgs)) != 0) {
+    const bool caches_changed = !h->args_valid || std::memcmp(a.k_cache, h->h_args.k_cache, sizeof(a.k_cache)) != 0 ||
+                                std::memcmp(a.v_cache, h->h_args.v_cache, sizeof(a.v_cache)) != 0;
     h->h_args = a;
     FSX_CUDA(cudaMemcpyAsync(h->d_args, &h->h_args, sizeof(TickArgs), cudaMemcpyHostToDevice, st));
+    if (caches_changed && h->d_cache_maps != nullptr) {
+      // the map of a NULL pointer stays zero: a layer without cache rows never loads through it
+      std::memset(h->h_cache_maps.data(), 0, h->h_cache_maps.size() * sizeof(CUtensorMap));
+      for (int l = 0; l < h->cfg.n_layers; ++l)
+        for (int t = 0; t < 2; ++t) {
+          const void* base = t == 0 ? a.k_cache[l] : a.v_cache[l];
+          if (base != nullptr &&
+              !fsx::encode_cache_map(&h->h_cache_maps[2 * l + t], base,
+                                     static_cast<uint64_t>(h->cfg.max_total_cache_tokens), h->cfg.n_heads))
+            return fail(FSX_ERR_INVALID_ARG, "a cache pointer is not 16-byte aligned (tensor map encoding failed)");
+        }
+      FSX_CUDA(cudaMemcpyAsync(h->d_cache_maps, h->h_cache_maps.data(), h->h_cache_maps.size() * sizeof(CUtensorMap),
+                               cudaMemcpyHostToDevice, st));
+    }
     h->args_valid = true;
   }
   return FSX_OK;
@@ -481,7 +502,7 @@ void free_handle(fsx_handle_s* h) {
   if (h->paper_params) cudaFree(h->paper_params);
   if (h->paper_frames) cudaFree(h->paper_frames);
   void* bufs[] = {h->p_arena, h->p_x, h->p_counters, h->w_arena, h->params, h->x, h->x16, h->ss, h->qkv, h->o, h->hbuf, h->part,
-                  h->gemm_part, h->tile_count, h->order, h->plan, h->status, h->d_args,
+                  h->gemm_part, h->tile_count, h->order, h->plan, h->status, h->d_args, h->d_cache_maps,
                   h->st_offsets, h->st_frames, h->st_waypoints};
   for (void* p : bufs)
     if (p) cudaFree(p);
@@ -762,6 +783,10 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
   FSX_CUDA_H(cudaMalloc(&h->status, sizeof(int)));
   FSX_CUDA_H(cudaMemset(h->status, 0, sizeof(int)));
   FSX_CUDA_H(cudaMalloc(&h->d_args, sizeof(TickArgs)));
+  if (cfg->cache_dtype == FSX_BF16 && cfg->max_total_cache_tokens > 0 && cfg->max_total_cache_tokens <= INT32_MAX) {
+    h->h_cache_maps.resize(2 * static_cast<size_t>(cfg->n_layers));
+    FSX_CUDA_H(cudaMalloc(&h->d_cache_maps, h->h_cache_maps.size() * sizeof(CUtensorMap)));
+  }
   FSX_CUDA_H(cudaMalloc(&h->st_offsets, (cfg->max_batch + 1) * sizeof(int64_t)));
   FSX_CUDA_H(cudaMalloc(&h->st_frames, static_cast<size_t>(cfg->max_batch) * cfg->n_frame * d * sizeof(float) + 16));
   FSX_CUDA_H(cudaMalloc(&h->st_waypoints, static_cast<size_t>(cfg->max_batch) * cfg->n_waypoints * 2 * sizeof(float)));

@@ -54,5 +54,8 @@ cudaError_t launch_gemm_tc(const CUtensorMap& map_a, const TcGemmArgs& args, int
 void pack_tc_tile(const float* const* rows, const float* col_scale, int k0, __half* out);
 // 2-D fp16 tensor map over a row-major [rows, cols] buffer with a (box_rows x 64) box and 128-byte swizzle.
 bool encode_act_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
+// 3-D bf16 tensor map over a token-major KV cache [rows, n_heads, 128]: a box is 64 tokens of one
+// head and 64 of its 128 dims, 128-byte swizzle (the attention's operand layout).
+bool encode_cache_map(CUtensorMap* map, const void* base, uint64_t rows, uint32_t n_heads);
 
 }  // namespace fsx

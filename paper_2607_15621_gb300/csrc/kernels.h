@@ -2,6 +2,7 @@
 // kernel translation units. Not part of the public ABI.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -63,6 +64,9 @@ struct AttnArgs {
   float* part_lse;            // [B, H, S, 48]   (log2 domain)
   const int* order;           // optional [B]: CTA row z works on vehicle order[z] (longest cache first)
   const AttnPlan* plan;       // optional [B] (tensor-core path): CTA row z works on plan[z]
+  // optional (tensor-core path, with targs): [2 n_layers] TMA maps of the layers' K and V caches
+  // (bf16 [rows, n_heads, 128]); whole 64-key chunks are then loaded by TMA
+  const CUtensorMap* cache_maps;
   int* status;
 };
 
