@@ -477,14 +477,16 @@ __global__ void __launch_bounds__(kThreadsTc, 2) attn_tc_kernel(const AttnArgs p
           issued = i + 3;
         }
       }
-      if (i > 0 && !is_v) {  // cache K rows -> fp16 (V stays bf16)
+      if (i > 0 && !is_v) {  // cache K rows -> fp16 (V stays bf16): every read before the first write
         unsigned char* slot = pslots + (i % kSlots) * kSlotBytes;
-#pragma unroll 8
-        for (int m = 0; m < kSlotKeys / 4; ++m) {
-          uint4* ptr = reinterpret_cast<uint4*>(slot + tile128_off(pr0 + 4 * m, pu));
-          const uint4 v = *ptr;
-          *ptr = make_uint4(bf16x2_to_half2(v.x), bf16x2_to_half2(v.y), bf16x2_to_half2(v.z), bf16x2_to_half2(v.w));
-        }
+        uint4 v[kSlotKeys / 4];
+#pragma unroll
+        for (int m = 0; m < kSlotKeys / 4; ++m) v[m] = *reinterpret_cast<const uint4*>(slot + tile128_off(pr0 + 4 * m, pu));
+#pragma unroll
+        for (int m = 0; m < kSlotKeys / 4; ++m)
+          *reinterpret_cast<uint4*>(slot + tile128_off(pr0 + 4 * m, pu)) =
+              make_uint4(bf16x2_to_half2(v[m].x), bf16x2_to_half2(v[m].y), bf16x2_to_half2(v[m].z),
+                         bf16x2_to_half2(v[m].w));
       }
       fence_proxy_async();
       mbar_arrive(full + (i % kSlots));
