@@ -40,6 +40,8 @@ struct TcGemmArgs {
   int k_splits;
   float* part;
   int* tile_count;
+  // pair variant: index of the tile at `w` in the weight map (tiles of 16 KB from the map's base)
+  int w_tile0;
 };
 
 // k splits for a residual GEMM with `tiles` output tiles of KT k steps on `sm_count` SMs
@@ -48,8 +50,12 @@ int gemm_tc_k_splits(int tiles, int KT, int sm_count);
 size_t gemm_tc_part_bytes(int sm_count);
 
 cudaError_t gemm_tc_set_attributes();
+// co-resident CTA pairs of the pair variant on this device (0: the variant is not available)
+int gemm_tc_pair_clusters();
+// map_w != nullptr selects the pair variant (bn 256, RMSNorm-fused store epilogue, N a multiple
+// of 256, no K split): map_a then has 128-row boxes and map_w covers the packed weight tiles
 cudaError_t launch_gemm_tc(const CUtensorMap& map_a, const TcGemmArgs& args, int bn, int epi, bool norm,
-                           cudaStream_t stream, bool pdl);
+                           cudaStream_t stream, bool pdl, const CUtensorMap* map_w = nullptr);
 // rows[128]: pointers to the 128 source rows (fp32, length >= k0 + 64); col_scale: optional per-K gain.
 void pack_tc_tile(const float* const* rows, const float* col_scale, int k0, __half* out);
 // 2-D fp16 tensor map over a row-major [rows, cols] buffer with a (box_rows x 64) box and 128-byte swizzle.
@@ -57,5 +63,8 @@ bool encode_act_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
 // 3-D bf16 tensor map over a token-major KV cache [rows, n_heads, 128]: a box is 64 tokens of one
 // head and 64 of its 128 dims, 128-byte swizzle (the attention's operand layout).
 bool encode_cache_map(CUtensorMap* map, const void* base, uint64_t rows, uint32_t n_heads);
+// 3-D fp16 tensor map over `n_tiles` packed 16 KB weight tiles [tiles][128 rows][64], no swizzle:
+// a box is one whole tile image
+bool encode_weight_map(CUtensorMap* map, const void* base, uint64_t n_tiles);
 
 }  // namespace fsx

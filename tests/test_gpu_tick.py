@@ -88,6 +88,34 @@ def test_tick_bf16_b128_ragged_sampled():
     _parity(case, vehicles=pick)
 
 
+def test_pair_gemm_matches_single_cta_gemm(monkeypatch):
+    """B = 64 (M = 2688 tokens): QKV runs 256-token tiles on CTA pairs
+    (tcgen05.mma.cta_group::2) by default and on single CTAs with FSX_NO_PAIR_GEMM=1 (read
+    at handle creation). Both accumulate the same fp16 products in fp32 in the same K order:
+    the per-layer attention outputs and the waypoints agree to rounding, and the pair
+    variant's tick matches the oracle on sampled vehicles."""
+    case = fc.Case(SMALL, list(np.random.default_rng(11).integers(40, 400, 64)), "bf16", seed=11)
+    ex = case.expert()
+    try:
+        wp_pair, att_pair = fc.run_debug_tick(ex, case)
+        wp_pair_graph = fc.run_tick(ex, case)
+    finally:
+        ex.close()
+    monkeypatch.setenv("FSX_NO_PAIR_GEMM", "1")
+    ex = case.expert()
+    try:
+        wp_one, att_one = fc.run_debug_tick(ex, case)
+    finally:
+        ex.close()
+    assert np.array_equal(wp_pair_graph, wp_pair)
+    a1 = att_pair.float().cpu().numpy()
+    a2 = att_one.float().cpu().numpy()
+    assert np.max(np.abs(a1 - a2)) <= 1e-3 * np.max(np.abs(a2))
+    assert np.linalg.norm(wp_pair - wp_one) <= 1e-4 * np.linalg.norm(wp_one)
+    for b in (0, 37, 63):
+        fc.check_vehicle(case, b, wp_pair, att_pair)
+
+
 def test_cache_is_never_written_and_vehicles_are_independent():
     case = fc.Case(SMALL, [40, 90, 17], "bf16", seed=2)
     before = [(k.clone(), v.clone()) for k, v in zip(case.k, case.v)]
