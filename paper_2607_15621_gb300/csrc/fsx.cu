@@ -70,7 +70,7 @@ struct fsx_handle_s {
   // 2-D tensor maps of the activation buffers for the token tile sizes 48 / 128 / 256
   CUtensorMap map_x16[4], map_o[4], map_h[4];  // token boxes of 48, 128, 256, 144 rows
   CUtensorMap map_w;                            // every packed weight tile (pair GEMM variant)
-  bool pair_gemm = false;                       // QKV and gate/up at 256-token tiles run on CTA pairs
+  bool pair_gemm = false;                       // QKV at 256-token tiles may run on CTA pairs (opt-in)
   // fp32 small parameters
   float* params = nullptr;
   float *act_emb = nullptr, *pos_emb = nullptr, *attn_norm = nullptr, *mlp_norm = nullptr;
@@ -273,9 +273,9 @@ fsx_status enqueue_tick(fsx_handle_s* h, int B, cudaStream_t st, __half* attn_ca
   const int rtiles144 = (d / 128) * ((M + 143) / 144);
   const int rbn_i = (bn_i == 2 && rtiles144 <= h->sm_count) ? 3 : bn_i;
   const int rbn = rbn_i == 3 ? 144 : bn;
-  // QKV on CTA pairs (M = 256 tcgen05.mma.cta_group::2, half the token rows staged per SM):
-  // at 5376 tokens 68 us per launch against 73 on single CTAs, at 672 tokens 20.1 against 18.5
-  // us, so only from 2048 tokens on. (gate/up at 5376 tokens: 26.7 against 26.0 us, single.)
+  // QKV on CTA pairs (M = 256 tcgen05.mma.cta_group::2, half the token rows staged per SM)
+  // when opted in, from 2048 tokens on. With the TMA-store epilogue the single-CTA kernel is
+  // the faster one (5376 tokens: 60.7 against 67.3 us per launch), so it is the default.
   const bool qkv_pair = h->pair_gemm && bq == 256 && M >= 2048;
   const int S = attention_splits(h, B);
 
@@ -652,9 +652,10 @@ fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, f
     for (auto& th : pool) th.join();
     FSX_CUDA_H(cudaMemcpy(h->w_arena, host.data(), arena, cudaMemcpyHostToDevice));
   }
-  // the pair GEMM variant (CTA pairs on tcgen05.mma.cta_group::2) loads the weight tiles
-  // through one map over the whole arena; FSX_NO_PAIR_GEMM=1 keeps the single-CTA kernel
-  h->pair_gemm = fsx::gemm_tc_pair_clusters() > 0 && std::getenv("FSX_NO_PAIR_GEMM") == nullptr &&
+  // the pair GEMM variant (CTA pairs on tcgen05.mma.cta_group::2, opted into by
+  // FSX_PAIR_GEMM=1 at handle creation) loads the weight tiles through one map over the arena
+  const char* pair_env = std::getenv("FSX_PAIR_GEMM");
+  h->pair_gemm = fsx::gemm_tc_pair_clusters() > 0 && pair_env != nullptr && std::strcmp(pair_env, "1") == 0 &&
                  arena / tile <= 0x7fffffffull && fsx::encode_weight_map(&h->map_w, h->w_arena, arena / tile);
   for (int l = 0; l < L; ++l) {
     const unsigned char* base = static_cast<const unsigned char*>(h->w_arena) + per_layer * l;

@@ -23,7 +23,7 @@
 //     stmatrix, then stored as 16-byte row pieces; the fp32 residual update
 //     reads its 32 lanes in the 32x32b shape (each element owned by one thread)
 //     and also emits each token's sum of x^2 over its 128 columns.
-// Pair variant (QKV at 256-token tiles and 2048 tokens or more): a cluster of two CTAs on an SM
+// Pair variant (opt-in for QKV at 256-token tiles and 2048 tokens or more): a cluster of two CTAs on an SM
 // pair computes D[256 weight rows, 256 tokens] with tcgen05.mma.cta_group::2 (M = 256):
 // each CTA stages its own 128-row weight tile and half of the 256 token rows (32 KB per
 // stage instead of 48, so six stages fit instead of four), the even CTA issues the MMAs
@@ -51,7 +51,7 @@ constexpr int kTileN = 128;           // weight rows per tile (MMA M)
 constexpr int kTileK = 64;            // K per stage (128 bytes of fp16: one swizzle span)
 constexpr int kWTileBytes = kTileN * kTileK * 2;  // 16 KB
 constexpr int kEpiChunk = 32;                     // tokens per epilogue round of one half
-constexpr int kStgHalfBytes = 9216;               // fp16 staging of one group: 32 tokens x (128 + 8) halves
+constexpr int kStgHalfBytes = 8192;               // fp16 staging of one group: 32 tokens x 128 columns (two TMA boxes)
 constexpr int kSspBytes = ((kEpiGroups * 32 * 4 * 4 + 1023) / 1024) * 1024;  // x^2 partials [groups][32][4]
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
@@ -60,6 +60,13 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
           smem_addr(dst)),
       "l"(map), "r"(x), "r"(y), "r"(smem_addr(bar))
       : "memory");
+}
+
+// TMA store of a (64 columns x 32 rows) box of the output from 128-byte swizzled shared memory
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(map),
+               "r"(smem_addr(src)), "r"(x), "r"(y)
+               : "memory");
 }
 
 // Copies of the pair variant: they land in this CTA's shared memory and complete on the
@@ -181,6 +188,7 @@ __host__ __device__ constexpr uint32_t tc_tmem_cols() {  // two accumulators, po
 template <int BN, int EPI, bool NORM, bool PAIR>
 __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_constant__ CUtensorMap map_a,
                                                                const __grid_constant__ CUtensorMap map_w,
+                                                               const __grid_constant__ CUtensorMap map_y,
                                                                const TcGemmArgs p) {
   static_assert(!PAIR || (BN == 256 && EPI != kEpiResidual), "the pair variant runs 256-token store / SwiGLU tiles");
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -399,8 +407,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
     const int htid = etid & 127;
     const int q = warp & 3;
     const int row = q * 32 + lane;
-    constexpr int kSH = kTileN + 8;  // fp16 row stride (store)
-    constexpr int kSG = 64 + 8;      // fp16 row stride (SwiGLU: 64 columns per tile)
     __half* tH = reinterpret_cast<__half*>(stg + half * kStgHalfBytes);
     float* ssp = s_ssp + half * kEpiChunk * 4;
     // x[m, n0 + row] += D[row, m] for the chunk's tokens: lanes hold consecutive columns,
@@ -503,75 +509,65 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
           auto val = [&](int hh, int k) {  // element k of the fragment registers of half hh
             return __uint_as_float(hh == 0 ? ra[k] : rb[k]);
           };
+          // The chunk's fp16 outputs, 8x8 blocks as fragments: store -- weight rows
+          // 32q + 8nb .. (nb = 2hh + {0, 1}), tokens 8i ..; SwiGLU -- packed rows 16b .. 16b + 7
+          // are gate rows and 16b + 8 .. 16b + 15 their up rows, so a thread holds each gate
+          // value (fragment row g) beside its up value (row g + 8): output columns
+          // 8 (2q + hh) + g, tokens 8i + 2 fq (+1).
+          constexpr int kNF = EPI == kEpiStore ? 16 : 8;
+          uint32_t f[kNF];
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+              const float a0 = val(hh, 4 * i) * rs[i].x, a1 = val(hh, 4 * i + 1) * rs[i].y;
+              const float a2 = val(hh, 4 * i + 2) * rs[i].x, a3 = val(hh, 4 * i + 3) * rs[i].y;
+              if (EPI == kEpiStore) {
+                f[4 * i + 2 * hh] = pack_half2(a0, a1);
+                f[4 * i + 2 * hh + 1] = pack_half2(a2, a3);
+              } else {
+                f[2 * i + hh] =
+                    pack_half2(__fdividef(a0, 1.f + __expf(-a0)) * a2, __fdividef(a1, 1.f + __expf(-a1)) * a3);
+              }
+            }
+          // the group's staging tile is free once its previous TMA store has read it
+          if (htid == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+          half_sync(half);
+          // stmatrix (transposed) into the staging tile in the layout of the output TMA box:
+          // 64 columns x 32 tokens per 4 KB box, token row r at 128 r, 16-byte unit u at
+          // u ^ (r mod 8) (the 128-byte swizzle; the 8 rows of a matrix hit 8 bank groups)
+          const uint32_t sbase = smem_addr(tH);
+          const int tr = lane & 7;  // row of the matrix this lane addresses
           if (EPI == kEpiStore) {
-            // 8x8 blocks (weight rows 32q + 8nb .., tokens 8i ..) stored transposed into the
-            // token-major staging tile: one stmatrix per token block i
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-              uint32_t f[4];
-#pragma unroll
-              for (int hh = 0; hh < 2; ++hh) {
-                f[2 * hh] = pack_half2(val(hh, 4 * i) * rs[i].x, val(hh, 4 * i + 1) * rs[i].y);
-                f[2 * hh + 1] = pack_half2(val(hh, 4 * i + 2) * rs[i].x, val(hh, 4 * i + 3) * rs[i].y);
-              }
-              stsm_x4_trans(smem_addr(tH + (8 * i + (lane & 7)) * kSH + 32 * q + 8 * (lane >> 3)), f[0], f[1], f[2],
-                            f[3]);
+              const int tok = 8 * i + tr;
+              const int col = 32 * q + 8 * (lane >> 3);
+              const uint32_t a = sbase + (col >> 6) * 4096 + tok * 128 + ((((col & 63) >> 3) ^ (tok & 7)) << 4);
+              stsm_x4_trans(a, f[4 * i], f[4 * i + 1], f[4 * i + 2], f[4 * i + 3]);
             }
-          }
-          if (EPI == kEpiSwiglu) {
-            // packed rows 16b .. 16b + 7 are gate rows, 16b + 8 .. 16b + 15 their up rows, so a
-            // thread holds each gate value (fragment row g) beside its up value (row g + 8):
-            // output columns 8 (2q + hh) + g, tokens 8i + 2 fq (+1)
+          } else {
 #pragma unroll
             for (int ip = 0; ip < 2; ++ip) {
-              uint32_t f[4];
-#pragma unroll
-              for (int mi = 0; mi < 4; ++mi) {
-                const int hh = mi & 1, i = 2 * ip + (mi >> 1);
-                const float g0 = val(hh, 4 * i) * rs[i].x, g1 = val(hh, 4 * i + 1) * rs[i].y;
-                const float u0 = val(hh, 4 * i + 2) * rs[i].x, u1 = val(hh, 4 * i + 3) * rs[i].y;
-                f[mi] = pack_half2(__fdividef(g0, 1.f + __expf(-g0)) * u0, __fdividef(g1, 1.f + __expf(-g1)) * u1);
-              }
-              const int mi = lane >> 3;
-              stsm_x4_trans(smem_addr(tH + (8 * (2 * ip + (mi >> 1)) + (lane & 7)) * kSG + 8 * (2 * q + (mi & 1))), f[0],
-                            f[1], f[2], f[3]);
+              const int mi = lane >> 3;  // matrix mi: half mi & 1, token block 2 ip + mi / 2
+              const int tok = 8 * (2 * ip + (mi >> 1)) + tr;
+              const int u = 2 * q + (mi & 1);
+              stsm_x4_trans(sbase + tok * 128 + ((u ^ (tok & 7)) << 4), f[4 * ip], f[4 * ip + 1], f[4 * ip + 2],
+                            f[4 * ip + 3]);
             }
           }
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // staging -> TMA store
           half_sync(half);
-          // coalesced 16-byte stores of the chunk's token rows
-          // (all of a thread's staging reads before its first global store)
-          if (EPI == kEpiStore) {  // 32 tokens x 16 units: four per thread
-            uint4 val[4];
-#pragma unroll
-            for (int t = 0; t < 4; ++t) {
-              const int e = htid + t * 128;
-              val[t] = *reinterpret_cast<const uint4*>(tH + (e >> 4) * kSH + (e & 15) * 8);
+          // one thread stores the chunk's token rows (rows past M are clipped by the map)
+          if (htid == 0 && m0 + c0 < p.M) {
+            if (EPI == kEpiStore) {
+              tma_store_2d(&map_y, tH, n0, m0 + c0);
+              tma_store_2d(&map_y, reinterpret_cast<const unsigned char*>(tH) + 4096, n0 + 64, m0 + c0);
+            } else {
+              tma_store_2d(&map_y, tH, n0 / 2, m0 + c0);
             }
-#pragma unroll
-            for (int t = 0; t < 4; ++t) {
-              const int e = htid + t * 128;
-              const int tk = e >> 4;
-              const int m = m0 + c0 + tk;
-              if (tk < nc && m < p.M)
-                *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m) * p.ldy + n0 + (e & 15) * 8) = val[t];
-            }
-          } else {  // 32 tokens x 8 units: two per thread
-            uint4 val[2];
-#pragma unroll
-            for (int t = 0; t < 2; ++t) {
-              const int e = htid + t * 128;
-              val[t] = *reinterpret_cast<const uint4*>(tH + (e >> 3) * kSG + (e & 7) * 8);
-            }
-#pragma unroll
-            for (int t = 0; t < 2; ++t) {
-              const int e = htid + t * 128;
-              const int tk = e >> 3;
-              const int m = m0 + c0 + tk;
-              if (tk < nc && m < p.M)
-                *reinterpret_cast<uint4*>(p.y + static_cast<size_t>(m) * p.ldy + n0 / 2 + (e & 7) * 8) = val[t];
-            }
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
           }
-          half_sync(half);  // staging free for the next chunk
         }
       }
       // accumulator drained: hand it back to the MMA warp (pair: the even CTA's)
@@ -658,6 +654,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
         if (etid == 0 && atomicAdd(p.tile_count + tile, 1) == 2 * KS - 1) p.tile_count[tile] = 0;
       }
     }
+    // the output stores of this group complete before the CTA leaves
+    if (EPI != kEpiResidual && htid == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   }
   tc_fence_before();
   __syncthreads();
@@ -781,8 +779,18 @@ cudaError_t launch_gemm_tc(const CUtensorMap& map_a, const TcGemmArgs& args, int
   CUtensorMap map = map_a;
   CUtensorMap mapw{};
   if (pair) mapw = *map_w;
+  // the store and SwiGLU epilogues write their output rows by TMA: a map over y[M, cols]
+  // (row stride ldy) with 64-column x 32-token boxes in the 128-byte swizzle
+  CUtensorMap mapy{};
+  if (epi != kEpiResidual) {
+    const int cols = epi == kEpiStore ? args.N : args.N / 2;
+    if (args.y == nullptr || args.M <= 0 || (reinterpret_cast<uintptr_t>(args.y) & 15) != 0 || (args.ldy * 2) % 16 != 0 ||
+        cols % 64 != 0 || args.ldy < cols || !encode_out_map(&mapy, args.y, static_cast<uint64_t>(args.M),
+                                                             static_cast<uint64_t>(cols), static_cast<uint64_t>(args.ldy)))
+      return cudaErrorInvalidValue;
+  }
   TcGemmArgs a = args;
-  void* kargs[] = {&map, &mapw, &a};
+  void* kargs[] = {&map, &mapw, &mapy, &a};
   if (a.k_splits > 1 && (epi != kEpiResidual || a.part == nullptr || a.tile_count == nullptr)) return cudaErrorInvalidValue;
   const int units = (args.N / kTileN) * ((args.M + bn - 1) / bn) * (a.k_splits > 1 ? a.k_splits : 1);
   if (pair) {  // one cluster of two CTAs per pair unit, at most as many as are co-resident
@@ -838,6 +846,18 @@ bool encode_act_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
   const cuuint64_t dims[2] = {cols, rows};
   const cuuint64_t strides[1] = {cols * 2};
   const cuuint32_t box[2] = {static_cast<cuuint32_t>(kTileK), box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_out_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld) {
+  const EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {ld * 2};
+  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(kEpiChunk)};
   const cuuint32_t estr[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,

@@ -63,6 +63,9 @@ bool encode_act_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
 // 3-D bf16 tensor map over a token-major KV cache [rows, n_heads, 128]: a box is 64 tokens of one
 // head and 64 of its 128 dims, 128-byte swizzle (the attention's operand layout).
 bool encode_cache_map(CUtensorMap* map, const void* base, uint64_t rows, uint32_t n_heads);
+// 2-D fp16 tensor map over an output y[rows, cols] with row stride `ld` elements, 64-column x
+// 32-row boxes, 128-byte swizzle (the store / SwiGLU epilogues' TMA stores)
+bool encode_out_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld);
 // 3-D fp16 tensor map over `n_tiles` packed 16 KB weight tiles [tiles][128 rows][64], no swizzle:
 // a box is one whole tile image
 bool encode_weight_map(CUtensorMap* map, const void* base, uint64_t n_tiles);

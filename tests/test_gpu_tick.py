@@ -89,19 +89,19 @@ def test_tick_bf16_b128_ragged_sampled():
 
 
 def test_pair_gemm_matches_single_cta_gemm(monkeypatch):
-    """B = 64 (M = 2688 tokens): QKV runs 256-token tiles on CTA pairs
-    (tcgen05.mma.cta_group::2) by default and on single CTAs with FSX_NO_PAIR_GEMM=1 (read
-    at handle creation). Both accumulate the same fp16 products in fp32 in the same K order:
+    """B = 64 (M = 2688 tokens): QKV runs 256-token tiles on single CTAs by default and on
+    CTA pairs (tcgen05.mma.cta_group::2) with FSX_PAIR_GEMM=1 (read at handle creation). Both accumulate the same fp16 products in fp32 in the same K order:
     the per-layer attention outputs and the waypoints agree to rounding, and the pair
     variant's tick matches the oracle on sampled vehicles."""
     case = fc.Case(SMALL, list(np.random.default_rng(11).integers(40, 400, 64)), "bf16", seed=11)
+    monkeypatch.setenv("FSX_PAIR_GEMM", "1")
     ex = case.expert()
     try:
         wp_pair, att_pair = fc.run_debug_tick(ex, case)
         wp_pair_graph = fc.run_tick(ex, case)
     finally:
         ex.close()
-    monkeypatch.setenv("FSX_NO_PAIR_GEMM", "1")
+    monkeypatch.delenv("FSX_PAIR_GEMM")
     ex = case.expert()
     try:
         wp_one, att_one = fc.run_debug_tick(ex, case)
