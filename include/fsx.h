@@ -99,7 +99,11 @@ typedef struct {
 /* Create a handle on `device`: validates cfg (host), uploads fp16 weights in
  * the kernels' tile order, allocates workspace for cfg->max_batch vehicles.
  * Blocking. Errors: INVALID_ARG (null/negative fields), UNSUPPORTED (shape),
- * OOM, CUDA. Env FSX_TEST_FAIL_ALLOC=1 forces the OOM path (tests). */
+ * OOM, CUDA. Env FSX_TEST_FAIL_ALLOC=1 forces the OOM path (tests);
+ * FSX_PAIR_GEMM=1 runs the batched QKV projection (2048 tokens or more) on CTA
+ * pairs (tcgen05.mma.cta_group::2) instead of single CTAs, with the same
+ * results to rounding; FSX_DISABLE_PERSISTENT=1 (read at every tick) runs a
+ * single vehicle through the batched graph instead of the one-launch tick. */
 fsx_status fsx_create(const fsx_config* cfg, const fsx_weights* w, int device, fsx_handle* out);
 
 /* One expert tick for B vehicles (Sec. 3.1, Eq. 1; Sec. 3.3: the cache is read

@@ -90,9 +90,10 @@ def test_tick_bf16_b128_ragged_sampled():
 
 def test_pair_gemm_matches_single_cta_gemm(monkeypatch):
     """B = 64 (M = 2688 tokens): QKV runs 256-token tiles on single CTAs by default and on
-    CTA pairs (tcgen05.mma.cta_group::2) with FSX_PAIR_GEMM=1 (read at handle creation). Both accumulate the same fp16 products in fp32 in the same K order:
-    the per-layer attention outputs and the waypoints agree to rounding, and the pair
-    variant's tick matches the oracle on sampled vehicles."""
+    CTA pairs (tcgen05.mma.cta_group::2) with FSX_PAIR_GEMM=1 (read at handle creation).
+    Both accumulate the same fp16 products in fp32 in the same K order: the per-layer
+    attention outputs and the waypoints agree to rounding, and the pair variant's tick
+    matches the oracle on sampled vehicles."""
     case = fc.Case(SMALL, list(np.random.default_rng(11).integers(40, 400, 64)), "bf16", seed=11)
     monkeypatch.setenv("FSX_PAIR_GEMM", "1")
     ex = case.expert()
